@@ -1,0 +1,430 @@
+#!/usr/bin/env python3
+"""Benchmark of the ADPSGD hot path on GB300: one JSON line on stdout.
+
+A step is one whole ADPSGD run of the resnet18-n8 workload (n = 8 replicas of a
+ResNet-18-sized fp32 vector, P = 11,689,512; 2000 iterations; step size 0.1, x0.1 at
+iterations 1000 and 1500; momentum 0.9, weight decay 5e-4, noise sigma 1; Algorithm 2 with
+p_init = 4 and K_s = 500): every iteration one fused local-step launch over all replicas,
+every sync one fused average + variance launch, the period rule on the host.  Inputs are
+resident in HBM when the timed region starts (x and v are reset to x0 = 0 inside it);
+x and v (748 MB) are larger than L2, so no flush is needed between steps.
+
+value      replica-params/s of the whole run (n * P * iterations / step time), all ranks
+e2e        the same through the C ABI with host buffers: H2D of x0, v0, h, c and D2H of the
+           final x inside the timed region
+roofline   the local-step kernel (the dominant one): algorithmic bytes per launch
+           (16 n P + 8 P) over its mean CUDA-event duration, against the measured HBM copy
+           bandwidth; avg_variance reports the averaging kernel the same way (8 n P + 8 P)
+cpu_baseline  the CPU oracle on a bounded sample of the same workload, one host core
+
+--impl reference times the CPU oracle itself (the only reference this build has) on bounded
+samples of the same workload.  Under torchrun every rank runs its own independent problem
+(weak scaling; the path has no cross-rank exchange) and rank 0 prints the max-over-ranks time.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "avg+variance GB/s vs HBM peak; fused local-step replica-params/sec"
+UNIT = "replica-params/s"
+CPU_SAMPLE_COLUMNS = 1 << 20
+CPU_SAMPLE_ITERS = 8
+
+
+def log(*a):
+    print(*a, file=sys.stderr, flush=True)
+
+
+def measured_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        with open(path) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    return 6800.0, "fallback"
+
+
+def recorded_traffic(kernel: str, workload: str):
+    """DRAM bytes per launch from a committed ncu capture, if the kernel source is unchanged since."""
+    path = os.path.join(ROOT, "profiles", "traffic.json")
+    if not os.path.exists(path):
+        return None
+    import hashlib
+    with open(path) as f:
+        d = json.load(f)
+    src = os.path.join(ROOT, "paper_2007_06134_gb300", "csrc", "kernels.cu")
+    digest = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
+    e = d.get(kernel, {}).get(workload)
+    if not e or e.get("kernels_cu_sha256_16") != digest:
+        return None
+    return e["dram_bytes_per_launch"]
+
+
+# ------------------------------------------------------------------------------------------
+# clocks during the timed region
+# ------------------------------------------------------------------------------------------
+
+class ClockSampler:
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,clocks_event_reasons.hw_slowdown,"
+              "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+              "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_id: str):
+        self.gpu_id = gpu_id
+        self.proc = None
+        self.path = os.path.join("/tmp", f"adpsgd_clocks_{os.getpid()}.csv")
+
+    def __enter__(self):
+        try:
+            self.f = open(self.path, "w")
+            self.proc = subprocess.Popen(["nvidia-smi", f"--id={self.gpu_id}", f"--query-gpu={self.FIELDS}",
+                                          "--format=csv,noheader,nounits", "-lms", "200"], stdout=self.f,
+                                         stderr=subprocess.DEVNULL)
+        except Exception as e:  # nvidia-smi missing: report no clock data
+            log("clock sampling unavailable:", e)
+            self.proc = None
+        return self
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+            self.f.close()
+
+    def summary(self):
+        if self.proc is None or not os.path.exists(self.path):
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"]}
+        sm, smax, reasons = [], [], set()
+        names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+        with open(self.path) as f:
+            for line in f:
+                parts = [p.strip() for p in line.split(",")]
+                if len(parts) < 8:
+                    continue
+                try:
+                    sm.append(float(parts[0]))
+                    smax.append(float(parts[1]))
+                except ValueError:
+                    continue
+                for nm, val in zip(names, parts[4:8]):
+                    if val.lower().startswith("active"):
+                        reasons.add(nm)
+        os.remove(self.path)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"]}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(smax), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# ------------------------------------------------------------------------------------------
+# distributed plumbing (barrier + max over ranks only; no data-path collective)
+# ------------------------------------------------------------------------------------------
+
+def dist_setup(args):
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    pg = None
+    if world > 1:
+        import torch.distributed as dist
+        backend = "nccl" if args.impl == "gb300" else "gloo"
+        if backend == "nccl":
+            import torch
+            torch.cuda.set_device(local)
+        dist.init_process_group(backend)
+        pg = dist
+    return world, rank, local, pg
+
+
+def max_over_ranks(pg, value: float, device=None) -> float:
+    if pg is None:
+        return value
+    import torch
+    t = torch.tensor([value], dtype=torch.float64, device=device)
+    pg.all_reduce(t, op=pg.ReduceOp.MAX)
+    return float(t.item())
+
+
+def barrier(pg, device=None):
+    if pg is not None:
+        if device is not None:
+            pg.barrier(device_ids=[device.index])
+        else:
+            pg.barrier()
+
+
+# ------------------------------------------------------------------------------------------
+# CPU oracle leg
+# ------------------------------------------------------------------------------------------
+
+def oracle_sample(w, seed_offset=0):
+    """Time the oracle on a bounded sample: CPU_SAMPLE_ITERS iterations of the workload's local step
+    and its syncs (constant period 4) on its first CPU_SAMPLE_COLUMNS columns, all replicas."""
+    from oracle import oracle as O
+    from paper_2007_06134_gb300 import inputs
+    P = min(CPU_SAMPLE_COLUMNS, w.P)
+    h, c = inputs.problem(w, P)
+    x, v = inputs.zero_state(w.n, P)
+    noise = O.noise_bf16(w.seed, w.n, P) if w.noise == "bf16" else None
+    spec = O.ScheduleSpec(kind=0, K=CPU_SAMPLE_ITERS, p_init=4, lr0=w.lr0, lr_factor=w.lr_factor,
+                          milestones=w.milestones)
+    O.build()
+    t0 = time.perf_counter()
+    O.run(x, v, h, c, spec=spec, seed=w.seed + seed_offset, mu=w.mu, wd=w.wd, sigma=w.sigma, noise=noise)
+    dt = time.perf_counter() - t0
+    rp = w.n * P * CPU_SAMPLE_ITERS
+    return rp / dt, dt, (f"{CPU_SAMPLE_ITERS} iterations (syncs every 4) of {w.name} on its first {P} columns, "
+                         f"all {w.n} replicas: {rp} replica-param updates in {dt:.2f} s")
+
+
+def run_reference(args, w):
+    world, rank, local, pg = dist_setup(args)
+    if rank != 0:
+        return 0
+    for _ in range(args.warmup):
+        oracle_sample(w)
+    rates, times, sample = [], [], ""
+    for s in range(args.steps):
+        r, dt, sample = oracle_sample(w, s + 1)
+        rates.append(r)
+        times.append(dt)
+    value = float(np.mean(rates))
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1000.0 * float(np.mean(times)),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+        "config": {"workload": w.name, "n": w.n, "P": w.P, "K": w.K, "sample_columns": min(CPU_SAMPLE_COLUMNS, w.P),
+                   "sample_iterations": CPU_SAMPLE_ITERS},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": sample},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+# ------------------------------------------------------------------------------------------
+# GPU leg
+# ------------------------------------------------------------------------------------------
+
+def schedule_for(abi, w):
+    return abi.make_schedule(abi.ADPSGD, w.K, w.p_init, K_s=w.K_s, lr0=w.lr0, lr_factor=w.lr_factor,
+                             milestones=w.milestones)
+
+
+def run_gpu(args, w):
+    import torch
+
+    from paper_2007_06134_gb300 import abi, inputs
+
+    world, rank, local, pg = dist_setup(args)
+    device = torch.device("cuda", local)
+    torch.cuda.set_device(device)
+    stream = torch.cuda.current_stream(device)
+    abi.load()
+    seed = w.seed + rank  # independent problem per rank
+
+    h, c = inputs.problem(w)
+    n, P = w.n, w.P
+    hd = torch.from_numpy(h).to(device)
+    cd = torch.from_numpy(c).to(device)
+    xd = torch.zeros((n, P), dtype=torch.float32, device=device)
+    vd = torch.zeros_like(xd)
+    noise = None
+    if w.noise == "bf16":
+        noise = torch.empty((n, P), dtype=torch.int16, device=device)
+        abi.adpsgd_noise_fill_bf16(w.seed, n, P, noise, stream)
+    cfg = abi.make_config(n, P, momentum=w.mu, weight_decay=w.wd, noise_sigma=w.sigma, seed=seed,
+                          noise_mode=abi.NOISE_BF16 if noise is not None else abi.NOISE_PHILOX, want_loss=True,
+                          time_kernels=True)
+    sched = schedule_for(abi, w)
+    ctx = abi.adpsgd_init(cfg, xd, vd, hd, cd, noise, stream)
+
+    def one_run():
+        xd.zero_()
+        vd.zero_()
+        st = abi.adpsgd_state_init(sched)
+        return abi.adpsgd_run(ctx, sched, st)
+
+    for _ in range(args.warmup):
+        stats = one_run()
+    abi.adpsgd_reset_kernel_times(ctx)
+    torch.cuda.synchronize(device)
+
+    gpu_id = str(local)
+    try:
+        gpu_id = str(torch.cuda.get_device_properties(device).uuid)
+        if not gpu_id.startswith("GPU-"):
+            gpu_id = "GPU-" + gpu_id
+    except Exception:
+        pass
+    ev0 = torch.cuda.Event(enable_timing=True)
+    ev1 = torch.cuda.Event(enable_timing=True)
+    rounds, launches = [], 0
+    with ClockSampler(gpu_id) as clocks:
+        barrier(pg, device)
+        torch.cuda.synchronize(device)
+        ev0.record(stream)
+        for _ in range(args.steps):
+            stats = one_run()
+            rounds.append(stats.rounds)
+            launches += stats.local_step_launches + 2 * stats.average_launches  # averaging = 2 kernels
+        ev1.record(stream)
+        torch.cuda.synchronize(device)
+        barrier(pg, device)
+    ms_total = ev0.elapsed_time(ev1)
+    ms_total = max_over_ranks(pg, ms_total, device)
+    ms_step = ms_total / args.steps
+    rp_per_step = n * P * w.K
+    value = world * rp_per_step / (ms_step / 1000.0)
+
+    kt = abi.adpsgd_kernel_times(ctx)
+    peak, peak_kind = measured_peaks()
+    k1_bytes = 16 * n * P + 8 * P + (2 * n * P if noise is not None else 0)
+    k1_ms = kt["local_step_ms"] / max(1, kt["local_step_launches"])
+    k1_gbs = k1_bytes / (k1_ms / 1000.0) / 1e9
+    k2_bytes = 8 * n * P + 8 * P
+    k2_ms = kt["average_ms"] / max(1, kt["average_launches"])
+    k2_gbs = k2_bytes / (k2_ms / 1000.0) / 1e9
+    clock_summary = clocks.summary()
+
+    # end to end through the C ABI from pinned host buffers
+    e2e_value, h2d, d2h = None, 0, 0
+    if not args.no_e2e:
+        x0h = torch.zeros((n, P), dtype=torch.float32).pin_memory()
+        v0h = torch.zeros_like(x0h).pin_memory()
+        hh = torch.from_numpy(h).pin_memory()
+        ch = torch.from_numpy(c).pin_memory()
+        xout = torch.empty_like(x0h).pin_memory()
+        h2d = 4 * (2 * n * P + 2 * P)
+        d2h = 4 * n * P
+        cfg_e2e = abi.make_config(n, P, momentum=w.mu, weight_decay=w.wd, noise_sigma=w.sigma, seed=seed,
+                                  noise_mode=cfg.noise_mode, want_loss=True)
+
+        def e2e_step():
+            xd.copy_(x0h, non_blocking=True)
+            vd.copy_(v0h, non_blocking=True)
+            hd.copy_(hh, non_blocking=True)
+            cd.copy_(ch, non_blocking=True)
+            with abi.adpsgd_init(cfg_e2e, xd, vd, hd, cd, noise, stream) as c2:
+                abi.adpsgd_run(c2, sched, abi.adpsgd_state_init(sched))
+            xout.copy_(xd, non_blocking=True)
+
+        e2e_step()
+        torch.cuda.synchronize(device)
+        barrier(pg, device)
+        t0 = time.perf_counter()
+        e2e_steps = max(1, min(args.steps, 3))
+        for _ in range(e2e_steps):
+            e2e_step()
+        torch.cuda.synchronize(device)
+        dt = max_over_ranks(pg, (time.perf_counter() - t0) / e2e_steps, device)
+        e2e_value = world * rp_per_step / dt
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu:
+        r, dt, sample = oracle_sample(w)
+        cpu = {"value": r, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": sample}
+    ctx.close()
+
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+            "config": {"workload": w.name, "n": n, "P": P, "K": w.K, "schedule": f"ADPSGD p_init={w.p_init} K_s={w.K_s}",
+                       "rounds_per_step": rounds[-1] if rounds else None,
+                       "l2": "inputs larger than L2 (x, v = %.0f MB)" % (8 * n * P / 1e6),
+                       "parallelism": f"independent problem per rank x{world}"},
+            "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
+            "gpu_launches": launches,
+            "roofline": {"kernel": "local_step_kernel", "bound": "hbm", "achieved": k1_gbs, "peak": peak,
+                         "peak_kind": peak_kind, "unit": "GB/s", "frac": k1_gbs / peak,
+                         "bytes_per_launch": k1_bytes, "ms_per_launch": k1_ms,
+                         "traffic": recorded_traffic("local_step_kernel", w.name)},
+            "avg_variance": {"kernel": "average_kernel+finalize_kernel", "bound": "hbm", "achieved": k2_gbs,
+                             "peak": peak, "unit": "GB/s", "frac": k2_gbs / peak, "bytes_per_launch": k2_bytes,
+                             "ms_per_launch": k2_ms, "launches": kt["average_launches"],
+                             "traffic": recorded_traffic("average_kernel", w.name)},
+            "local_step_rp_per_s": n * P / (k1_ms / 1000.0),
+            "clocks": clock_summary,
+            "cpu_baseline": cpu,
+        }
+        print(json.dumps(line), flush=True)
+    if pg is not None:
+        pg.destroy_process_group()
+    return 0
+
+
+def run_sweep(args):
+    """Averaging + variance alone over n x P (the sweep workload): GB/s and fraction of peak per point."""
+    import torch
+
+    from paper_2007_06134_gb300 import abi, inputs
+    peak, peak_kind = measured_peaks()
+    device = torch.device("cuda", 0)
+    stream = torch.cuda.current_stream(device)
+    l2 = torch.cuda.get_device_properties(device).L2_cache_size
+    flush = torch.empty(int(2 * l2) // 4, dtype=torch.float32, device=device)
+    for n in inputs.SWEEP_N:
+        for lp in inputs.SWEEP_LOG2P:
+            P = 1 << lp
+            if 8 * n * P > args.sweep_max_bytes:
+                continue
+            xd = torch.randn((n, P), dtype=torch.float32, device=device)
+            xd += torch.arange(n, device=device, dtype=torch.float32)[:, None] * 1e-3
+            z = torch.zeros(P, device=device)
+            cfg = abi.make_config(n, P, want_loss=False, time_kernels=True)
+            with abi.adpsgd_init(cfg, xd, xd, z, z, None, stream) as ctx:
+                reps = max(5, min(50, int(2e10 // (8 * n * P))))
+                for _ in range(3):
+                    abi.adpsgd_average_and_variance(ctx, want_loss=False)
+                abi.adpsgd_reset_kernel_times(ctx)
+                for _ in range(reps):
+                    flush.zero_()
+                    abi.adpsgd_average_and_variance(ctx, want_loss=False)
+                t = abi.adpsgd_kernel_times(ctx)
+            ms = t["average_ms"] / t["average_launches"]
+            gbs = 8 * n * P / (ms / 1e3) / 1e9
+            print(json.dumps({"sweep": "average_and_variance", "n": n, "P": P, "ms": ms, "GB/s": gbs,
+                              "frac": gbs / peak, "peak": peak, "peak_kind": peak_kind,
+                              "l2_flushed": True}), flush=True)
+            del xd
+
+
+def main():
+    ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=5)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=["gb300", "reference"], default="gb300")
+    ap.add_argument("--workload", default="resnet18-n8")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu", action="store_true")
+    ap.add_argument("--sweep", action="store_true", help="averaging-kernel sweep over n x P instead")
+    ap.add_argument("--sweep-max-bytes", type=float, default=34e9)
+    args = ap.parse_args()
+    from paper_2007_06134_gb300 import inputs
+    w = inputs.WORKLOADS[args.workload]
+    if args.impl == "reference":
+        return run_reference(args, w)
+    if args.sweep:
+        return run_sweep(args)
+    return run_gpu(args, w)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

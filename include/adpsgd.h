@@ -1,0 +1,221 @@
+/*
+ * adpsgd.h -- C ABI of the GB300 (sm_103a) data-parallel hot path of ADPSGD,
+ * adaptive periodic parameter averaging SGD (Jiang & Agrawal, "Adaptive
+ * Periodic Averaging: A Practical Approach to Reducing Communication in
+ * Distributed Learning", arXiv 2007.06134).
+ *
+ * n worker replicas ("nodes" in the paper) live on one GPU as an [n, P] fp32
+ * row-major tensor x (replica i at x + i*P) with momentum buffers v of the
+ * same shape.  The objective is the separable quadratic
+ *     f(x) = 1/2 sum_j h_j (x_j - c_j)^2
+ * standing in for the paper's CNN losses (Sec. II-A, Eq. obj1), with additive
+ * Gaussian gradient noise standing in for mini-batch sampling (Eq. eg).
+ *
+ * Conventions for every entry point:
+ *   - Pointers named x, v, h, c, noise, out are DEVICE pointers the caller owns
+ *     (allocated by the caller, e.g. through PyTorch); the library never frees
+ *     them and keeps only borrowed references inside a context.
+ *   - Pointers to structs and scalars (cfg, schedule, state, trace, stats,
+ *     D_out, lr, ...) are HOST pointers.
+ *   - `stream` is a cudaStream_t passed as void* (NULL = the legacy default
+ *     stream).  All device work is enqueued on it in order.
+ *   - Every call returns an adpsgd_status; no C++ exception crosses the ABI.
+ *     On ADPSGD_E_CUDA, adpsgd_last_error() gives the CUDA error text of the
+ *     calling thread.  Calls that return scalars to the host wait for them
+ *     with a bounded poll (cfg.wait_timeout_ms) and return ADPSGD_E_TIMEOUT
+ *     instead of blocking forever.
+ *   - Device pointers must be 16-byte aligned (ADPSGD_E_ALIGN otherwise);
+ *     P need not be a multiple of 4 (a scalar kernel variant handles that).
+ */
+#ifndef ADPSGD_H
+#define ADPSGD_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    ADPSGD_OK = 0,
+    ADPSGD_E_INVAL = -1,   /* an argument is out of range or NULL where it may not be */
+    ADPSGD_E_ALIGN = -2,   /* a device pointer is not 16-byte aligned */
+    ADPSGD_E_CUDA = -3,    /* a CUDA runtime call failed (see adpsgd_last_error) */
+    ADPSGD_E_TIMEOUT = -4, /* a bounded host wait ran out; the work may still be in flight */
+    ADPSGD_E_NOMEM = -5,   /* the context's own scratch could not be allocated */
+    ADPSGD_E_STATE = -6    /* call not valid in the current state (e.g. no noise tensor) */
+} adpsgd_status;
+
+/* Opaque context: borrowed pointers to x, v, h, c (and the noise tensor),
+ * the stream, and the only memory the library allocates itself: per-block
+ * fp64 partial sums on the device, two pinned host doubles, CUDA events. */
+typedef struct adpsgd_ctx adpsgd_ctx;
+
+enum { ADPSGD_NOISE_PHILOX = 0, ADPSGD_NOISE_BF16 = 1 };
+
+typedef struct {
+    int32_t n;               /* replicas, >= 1 (the paper's n nodes) */
+    int32_t noise_mode;      /* ADPSGD_NOISE_PHILOX: z drawn per step from Philox4x32-10;
+                                ADPSGD_NOISE_BF16: z read from a caller tensor [n, P] bf16 */
+    int64_t P;               /* parameters per replica, >= 1 */
+    float momentum;          /* mu (Sec. V-A uses 0.9) */
+    float weight_decay;      /* wd, added to the gradient as wd * x (0 = off) */
+    float noise_sigma;       /* sigma: g = h (x - c) + sigma z */
+    int32_t want_loss;       /* nonzero: averaging also returns 1/2 sum_j h_j (xbar_j - c_j)^2 */
+    uint64_t seed;           /* Philox key (low word, high word) */
+    int64_t wait_timeout_ms; /* bound on every host wait; <= 0 means 60000 */
+    int32_t time_kernels;    /* nonzero: bracket every kernel launch with CUDA events */
+    int32_t reserved;
+} adpsgd_config;
+
+/* Schedules (Algorithm 1: kind 0; Algorithm 2: kind 1). */
+enum { ADPSGD_CPSGD = 0, ADPSGD_ADPSGD = 1 };
+
+typedef struct {
+    int32_t kind;            /* ADPSGD_CPSGD (constant p) or ADPSGD_ADPSGD */
+    int32_t p_init;          /* the constant period, or Algorithm 2's p_init; >= 1 */
+    int64_t K;               /* total iterations of the schedule */
+    int64_t K_s;             /* Algorithm 2: syncs at iterations k < K_s sample C_2;
+                                must be >= p_init (+ K_w) so that C_2 gets a sample */
+    int64_t K_w;             /* warm-up: iterations k < K_w sync every iteration and are
+                                not sampled (Sec. V-B warm-up epoch); 0 = none */
+    double lo, hi;           /* Algorithm 2 thresholds, 0.7 and 1.3 in the paper */
+    int32_t p_min, p_max;    /* clamp of p after the rule; p_max = 0: no upper bound */
+    double lr0;              /* step size at k = 0 */
+    double lr_factor;        /* step size multiplied by this at each milestone */
+    int32_t n_milestones;    /* length of milestones[] (host array) */
+    int32_t literal_phase;   /* kind 0 only: sync when k mod p == 0 (Algorithm 1 as printed)
+                                instead of when cnt reaches p */
+    const int64_t* milestones; /* iterations from which the step size changes */
+} adpsgd_schedule;
+
+/* Scheduler state (everything besides x and v that a checkpoint needs). */
+typedef struct {
+    int64_t k_next;          /* next iteration to run */
+    int32_t cnt;             /* iterations since the last sync (Algorithm 2's cnt) */
+    int32_t p;               /* current period */
+    double C2;               /* sampled C_2 (cumulative mean of S_k / gamma_k) */
+    int64_t m;               /* number of samples in C2 */
+    int64_t rounds;          /* syncs so far */
+} adpsgd_state;
+
+/* Per-sync trace, caller-allocated host arrays of capacity cap. */
+typedef struct {
+    int64_t cap;             /* capacity of every array */
+    int64_t len;             /* entries written (<= cap); syncs beyond cap are counted, not stored */
+    int64_t* k;              /* iteration of the sync */
+    int32_t* p;              /* period after the rule ran */
+    double* S;               /* S_k = D / n */
+    double* C2;              /* C_2 after the rule ran */
+    double* loss;            /* 1/2 sum_j h_j (xbar_j - c_j)^2 (0 if want_loss == 0) */
+    int32_t* phase;          /* 0 constant, 1 warm-up, 2 sampling, 3 adapting */
+} adpsgd_trace;
+
+typedef struct {
+    int64_t rounds;                  /* syncs so far (state.rounds) */
+    double equiv_period;             /* k_next / rounds */
+    double wire_bytes_per_node;      /* ring allreduce of P fp32 + one fp32 S_k, per sync */
+    double wire_bytes_total;         /* times n */
+    double fullsgd_wire_bytes_per_node; /* one P-fp32 allreduce per iteration (FULLSGD) */
+    int64_t local_step_launches;     /* kernel launches issued by this call */
+    int64_t average_launches;
+} adpsgd_stats;
+
+/* Create a context over caller-owned device arrays.
+ * x, v: [n, P] fp32 (read/write); h, c: [P] fp32 (read only);
+ * noise_bf16: [n, P] bf16 (read only) when cfg->noise_mode == ADPSGD_NOISE_BF16, else NULL.
+ * The pointers must stay valid until adpsgd_destroy.  Errors: E_INVAL (bad n, P, NULL
+ * pointer, P*n overflow), E_ALIGN, E_NOMEM, E_CUDA.  On error *out is NULL. */
+int adpsgd_init(const adpsgd_config* cfg, float* x, float* v, const float* h, const float* c,
+                const uint16_t* noise_bf16, void* stream, adpsgd_ctx** out);
+
+/* m local steps of every replica (Algorithm 1 and 2, "updating parameter variables locally";
+ * Sec. V-A momentum): for t in [0, m), step k = k0 + t with step size lr[t] (host array):
+ *   g = h (x - c) + sigma z[i, j, k];  if wd != 0: g += wd x;  v = mu v + g;  x -= lr[t] v
+ * each a separately rounded fp32 operation.  z is word (j mod 4) of Philox4x32-10 with counter
+ * (j div 4, i, k, 0) and key (seed lo, seed hi), mapped through Box-Muller.  Enqueued only;
+ * does not wait.  Errors: E_INVAL (m < 0, k0 < 0, k0 + m > 2^32), E_CUDA. */
+int adpsgd_local_steps(adpsgd_ctx* ctx, int64_t k0, int32_t m, const float* lr);
+
+/* Synchronisation (Algorithm 2 averaging and S_k lines; Sec. III definition of Var[W_k]):
+ * for every column j, xbar_j = x_0j + (sum_{i>=1} (x_ij - x_0j)) / n in fp32, written back to
+ * all n replicas, and *D_out = sum_j sum_i (x_ij - xbar_j)^2 over the pre-average values
+ * (n * Var[W]), accumulated in fp64.  If loss_out != NULL (needs cfg.want_loss),
+ * *loss_out = 1/2 sum_j h_j (xbar_j - c_j)^2.  Blocks (bounded) until the scalars arrive.
+ * Errors: E_INVAL (D_out NULL), E_STATE (loss requested without want_loss), E_TIMEOUT, E_CUDA. */
+int adpsgd_average_and_variance(adpsgd_ctx* ctx, double* D_out, double* loss_out);
+
+/* D = sum_j sum_i (x_ij - xbar_j)^2 without averaging (the per-iteration Var[W_k] of
+ * Sec. III and Eq. vt, times n).  Blocks (bounded).  Errors: as above. */
+int adpsgd_variance(adpsgd_ctx* ctx, double* D_out);
+
+/* Initial scheduler state of a schedule: k_next 0, cnt 0, p = p_init, C2 0.  Errors: E_INVAL. */
+int adpsgd_state_init(const adpsgd_schedule* sched, adpsgd_state* state);
+
+/* Run iterations [state->k_next, min(k_end, sched->K)) of a schedule (Algorithm 2, or
+ * Algorithm 1 when kind == ADPSGD_CPSGD): each iteration one local step with gamma_k, then
+ * cnt += 1 and, when cnt reaches p, one averaging, S = D / n, and the period rule
+ * (adpsgd_sched_on_sync).  Updates *state so that a later call resumes bit-identically.
+ * trace and stats may be NULL.  Blocks (bounded) at every sync.  Errors: E_INVAL (bad
+ * schedule, K_s < p_init + K_w for kind 1, p < 1), E_TIMEOUT, E_CUDA. */
+int adpsgd_run(adpsgd_ctx* ctx, const adpsgd_schedule* sched, adpsgd_state* state, int64_t k_end,
+               adpsgd_trace* trace, adpsgd_stats* stats);
+
+/* The period rule alone (Algorithm 2, after the sync at iteration k; pure host code):
+ * warm-up (k < K_w) and kind 0 leave the state unchanged; k < K_s: m += 1,
+ * C2 += (S / gamma - C2) / m; otherwise p += 1 if S < lo * (gamma * C2), else p -= 1 if
+ * S > hi * (gamma * C2), then p is clamped to [p_min, p_max].  *phase (may be NULL)
+ * receives the phase code.  Errors: E_INVAL. */
+int adpsgd_sched_on_sync(const adpsgd_schedule* sched, adpsgd_state* state, int64_t k, double S,
+                         double gamma, int32_t* phase);
+
+/* Step size of iteration k: (float)(lr0 * lr_factor^(number of milestones <= k)), the product
+ * taken in fp64.  Errors: E_INVAL. */
+int adpsgd_gamma(const adpsgd_schedule* sched, int64_t k, float* gamma_out);
+
+/* Bytes a ring allreduce would move per node and in total for `rounds` syncs of P fp32
+ * values, 2 (n-1)/n * 4P each (plus 2 (n-1)/n * 4 for the fp32 S_k if with_scalar): the
+ * communication Algorithm 2 saves (Sec. V-B).  Errors: E_INVAL. */
+int adpsgd_wire_bytes(int32_t n, int64_t P, int64_t rounds, int32_t with_scalar,
+                      double* per_node, double* total);
+
+/* Raw Philox4x32-10 words of the noise stream: out[(i * nq + q) * 4 + r] = word r of
+ * Philox(counter (q, i, k, tag), key (seed lo, seed hi)), i < n, q < nq.  out: device
+ * uint32 [n, nq, 4].  Enqueued only.  Errors: E_INVAL, E_ALIGN, E_CUDA. */
+int adpsgd_philox_fill(uint64_t seed, uint32_t tag, int32_t n, int64_t nq, int64_t k,
+                       uint32_t* out, void* stream);
+
+/* The fp32 normals the local step uses: out[i * P + j] = z[i, j] of stream `tag` at step k
+ * (Box-Muller of words (0,1) -> elements 4q, 4q+1 and (2,3) -> 4q+2, 4q+3).  out: device fp32
+ * [n, P].  Enqueued only.  Errors: E_INVAL, E_ALIGN, E_CUDA. */
+int adpsgd_noise_fill_f32(uint64_t seed, uint32_t tag, int32_t n, int64_t P, int64_t k,
+                          float* out, void* stream);
+
+/* A pre-materialised bf16 noise tensor [n, P]: the step-0 normals of stream tag 1, rounded
+ * to nearest-even bf16.  out: device, raw bf16 bits.  Enqueued only.  Errors: as above. */
+int adpsgd_noise_fill_bf16(uint64_t seed, int32_t n, int64_t P, uint16_t* out, void* stream);
+
+/* Device time of the kernels launched through ctx while cfg.time_kernels was set, summed from
+ * CUDA events on ctx's stream since init or the last reset (waits for them, bounded).
+ * Any output pointer may be NULL.  Errors: E_STATE (timing off), E_TIMEOUT, E_CUDA. */
+int adpsgd_kernel_times(adpsgd_ctx* ctx, double* local_step_ms, int64_t* local_step_launches,
+                        double* average_ms, int64_t* average_launches);
+int adpsgd_reset_kernel_times(adpsgd_ctx* ctx);
+
+/* Test hook: when force_incomplete is nonzero every bounded wait of ctx behaves as if the
+ * awaited work never finished, so the wait returns ADPSGD_E_TIMEOUT after
+ * cfg.wait_timeout_ms.  Only for exercising the timeout path. */
+int adpsgd_test_force_incomplete(adpsgd_ctx* ctx, int32_t force_incomplete);
+
+/* Synchronise the context's stream (bounded) and release the context.  NULL is a no-op. */
+void adpsgd_destroy(adpsgd_ctx* ctx);
+
+/* Static text for a status code, and the calling thread's last CUDA error detail. */
+const char* adpsgd_strerror(int status);
+const char* adpsgd_last_error(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* ADPSGD_H */

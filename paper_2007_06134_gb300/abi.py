@@ -1,0 +1,322 @@
+"""ctypes binding of ``libadpsgd.so`` (include/adpsgd.h), one Python function per C entry point.
+
+Argument marshalling only: tensors become device pointers (``data_ptr()``), the stream
+becomes its ``cudaStream_t`` handle, and a nonzero status becomes an ``AdpsgdError``.
+Every step of the hot path runs in the library's CUDA kernels; if the library cannot be
+built or loaded this module raises, it never falls back to another implementation.
+"""
+from __future__ import annotations
+
+import ctypes as C
+import os
+import re
+import threading
+
+from . import build as _build
+
+_lock = threading.Lock()
+_lib = None
+
+OK, E_INVAL, E_ALIGN, E_CUDA, E_TIMEOUT, E_NOMEM, E_STATE = 0, -1, -2, -3, -4, -5, -6
+NOISE_PHILOX, NOISE_BF16 = 0, 1
+CPSGD, ADPSGD = 0, 1
+PHASE_CONSTANT, PHASE_WARMUP, PHASE_SAMPLING, PHASE_ADAPTING = 0, 1, 2, 3
+
+
+class AdpsgdError(RuntimeError):
+    def __init__(self, status: int, where: str):
+        self.status = status
+        detail = last_error() if status == E_CUDA or status == E_TIMEOUT else ""
+        super().__init__(f"{where}: {strerror(status)} ({status}){': ' + detail if detail else ''}")
+
+
+class Config(C.Structure):
+    _fields_ = [("n", C.c_int32), ("noise_mode", C.c_int32), ("P", C.c_int64), ("momentum", C.c_float),
+                ("weight_decay", C.c_float), ("noise_sigma", C.c_float), ("want_loss", C.c_int32),
+                ("seed", C.c_uint64), ("wait_timeout_ms", C.c_int64), ("time_kernels", C.c_int32),
+                ("reserved", C.c_int32)]
+
+
+class Schedule(C.Structure):
+    _fields_ = [("kind", C.c_int32), ("p_init", C.c_int32), ("K", C.c_int64), ("K_s", C.c_int64),
+                ("K_w", C.c_int64), ("lo", C.c_double), ("hi", C.c_double), ("p_min", C.c_int32),
+                ("p_max", C.c_int32), ("lr0", C.c_double), ("lr_factor", C.c_double),
+                ("n_milestones", C.c_int32), ("literal_phase", C.c_int32),
+                ("milestones", C.POINTER(C.c_int64))]
+
+
+class State(C.Structure):
+    _fields_ = [("k_next", C.c_int64), ("cnt", C.c_int32), ("p", C.c_int32), ("C2", C.c_double),
+                ("m", C.c_int64), ("rounds", C.c_int64)]
+
+
+class Trace(C.Structure):
+    _fields_ = [("cap", C.c_int64), ("len", C.c_int64), ("k", C.POINTER(C.c_int64)),
+                ("p", C.POINTER(C.c_int32)), ("S", C.POINTER(C.c_double)), ("C2", C.POINTER(C.c_double)),
+                ("loss", C.POINTER(C.c_double)), ("phase", C.POINTER(C.c_int32))]
+
+
+class Stats(C.Structure):
+    _fields_ = [("rounds", C.c_int64), ("equiv_period", C.c_double), ("wire_bytes_per_node", C.c_double),
+                ("wire_bytes_total", C.c_double), ("fullsgd_wire_bytes_per_node", C.c_double),
+                ("local_step_launches", C.c_int64), ("average_launches", C.c_int64)]
+
+
+_P = C.c_void_p
+_SIGS = {
+    "adpsgd_init": (C.c_int, [C.POINTER(Config), _P, _P, _P, _P, _P, _P, C.POINTER(_P)]),
+    "adpsgd_local_steps": (C.c_int, [_P, C.c_int64, C.c_int32, C.POINTER(C.c_float)]),
+    "adpsgd_average_and_variance": (C.c_int, [_P, C.POINTER(C.c_double), C.POINTER(C.c_double)]),
+    "adpsgd_variance": (C.c_int, [_P, C.POINTER(C.c_double)]),
+    "adpsgd_state_init": (C.c_int, [C.POINTER(Schedule), C.POINTER(State)]),
+    "adpsgd_run": (C.c_int, [_P, C.POINTER(Schedule), C.POINTER(State), C.c_int64, C.POINTER(Trace),
+                             C.POINTER(Stats)]),
+    "adpsgd_sched_on_sync": (C.c_int, [C.POINTER(Schedule), C.POINTER(State), C.c_int64, C.c_double,
+                                       C.c_double, C.POINTER(C.c_int32)]),
+    "adpsgd_gamma": (C.c_int, [C.POINTER(Schedule), C.c_int64, C.POINTER(C.c_float)]),
+    "adpsgd_wire_bytes": (C.c_int, [C.c_int32, C.c_int64, C.c_int64, C.c_int32, C.POINTER(C.c_double),
+                                    C.POINTER(C.c_double)]),
+    "adpsgd_philox_fill": (C.c_int, [C.c_uint64, C.c_uint32, C.c_int32, C.c_int64, C.c_int64, _P, _P]),
+    "adpsgd_noise_fill_f32": (C.c_int, [C.c_uint64, C.c_uint32, C.c_int32, C.c_int64, C.c_int64, _P, _P]),
+    "adpsgd_noise_fill_bf16": (C.c_int, [C.c_uint64, C.c_int32, C.c_int64, _P, _P]),
+    "adpsgd_kernel_times": (C.c_int, [_P, C.POINTER(C.c_double), C.POINTER(C.c_int64), C.POINTER(C.c_double),
+                                      C.POINTER(C.c_int64)]),
+    "adpsgd_reset_kernel_times": (C.c_int, [_P]),
+    "adpsgd_test_force_incomplete": (C.c_int, [_P, C.c_int32]),
+    "adpsgd_destroy": (None, [_P]),
+    "adpsgd_strerror": (C.c_char_p, [C.c_int]),
+    "adpsgd_last_error": (C.c_char_p, []),
+}
+
+
+def library_path() -> str:
+    return _build.LIB
+
+
+def load(build_if_stale: bool = True):
+    """Load (building first if needed) the CUDA library; raise if that is impossible."""
+    global _lib
+    with _lock:
+        if _lib is None:
+            if build_if_stale:
+                _build.build()
+            if not os.path.exists(_build.LIB):
+                raise RuntimeError(f"CUDA library missing: {_build.LIB} (build with paper_2007_06134_gb300.build)")
+            L = C.CDLL(_build.LIB)
+            for name, (res, args) in _SIGS.items():
+                f = getattr(L, name)
+                f.restype = res
+                f.argtypes = args
+            _lib = L
+    return _lib
+
+
+def header_entry_points() -> list[str]:
+    """Names of the functions include/adpsgd.h declares."""
+    hdr = os.path.join(_build.INCLUDE, "adpsgd.h")
+    text = open(hdr).read()
+    return sorted(set(re.findall(r"^\s*(?:int|void|const char\*)\s+(adpsgd_\w+)\s*\(", text, re.M)))
+
+
+def strerror(status: int) -> str:
+    return load().adpsgd_strerror(status).decode()
+
+
+def last_error() -> str:
+    return load().adpsgd_last_error().decode()
+
+
+def _check(status: int, where: str):
+    if status != OK:
+        raise AdpsgdError(status, where)
+
+
+def _ptr(t) -> int | None:
+    if t is None:
+        return None
+    if isinstance(t, int):
+        return t
+    return t.data_ptr()
+
+
+def _stream(stream) -> int | None:
+    if stream is None:
+        import torch
+        return torch.cuda.current_stream().cuda_stream
+    if isinstance(stream, int):
+        return stream
+    return stream.cuda_stream
+
+
+def make_config(n, P, *, momentum=0.9, weight_decay=0.0, noise_sigma=1.0, seed=0, noise_mode=NOISE_PHILOX,
+                want_loss=True, wait_timeout_ms=60000, time_kernels=False) -> Config:
+    return Config(n, noise_mode, P, momentum, weight_decay, noise_sigma, int(bool(want_loss)),
+                  seed & 0xFFFFFFFFFFFFFFFF, wait_timeout_ms, int(bool(time_kernels)), 0)
+
+
+def make_schedule(kind, K, p_init, *, K_s=0, K_w=0, lo=0.7, hi=1.3, p_min=1, p_max=0, lr0=0.1, lr_factor=0.1,
+                  milestones=(), literal_phase=False) -> Schedule:
+    ms = (C.c_int64 * max(1, len(milestones)))(*milestones)
+    s = Schedule(kind, p_init, K, K_s, K_w, lo, hi, p_min, p_max, lr0, lr_factor, len(milestones),
+                 int(bool(literal_phase)), C.cast(ms, C.POINTER(C.c_int64)))
+    s._keep = ms  # keep the milestone array alive with the struct
+    return s
+
+
+class Context:
+    """An ``adpsgd_ctx*`` over caller-owned device tensors; ``close()`` calls adpsgd_destroy."""
+
+    def __init__(self, handle: int, keep: tuple):
+        self.handle = handle
+        self._keep = keep  # tensors the context borrows
+
+    def close(self):
+        if self.handle:
+            load().adpsgd_destroy(self.handle)
+            self.handle = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    def __enter__(self):
+        return self
+
+    def __exit__(self, *exc):
+        self.close()
+
+
+def adpsgd_init(cfg: Config, x, v, h, c, noise_bf16=None, stream=None) -> Context:
+    out = C.c_void_p()
+    _check(load().adpsgd_init(C.byref(cfg), _ptr(x), _ptr(v), _ptr(h), _ptr(c), _ptr(noise_bf16),
+                              _stream(stream), C.byref(out)), "adpsgd_init")
+    return Context(out.value, (x, v, h, c, noise_bf16))
+
+
+def adpsgd_local_steps(ctx: Context, k0: int, lr) -> None:
+    lr = list(lr)
+    arr = (C.c_float * max(1, len(lr)))(*lr)
+    _check(load().adpsgd_local_steps(ctx.handle, k0, len(lr), arr), "adpsgd_local_steps")
+
+
+def adpsgd_average_and_variance(ctx: Context, want_loss: bool = True):
+    D = C.c_double()
+    L = C.c_double()
+    _check(load().adpsgd_average_and_variance(ctx.handle, C.byref(D), C.byref(L) if want_loss else None),
+           "adpsgd_average_and_variance")
+    return D.value, (L.value if want_loss else None)
+
+
+def adpsgd_variance(ctx: Context) -> float:
+    D = C.c_double()
+    _check(load().adpsgd_variance(ctx.handle, C.byref(D)), "adpsgd_variance")
+    return D.value
+
+
+def adpsgd_state_init(sched: Schedule) -> State:
+    st = State()
+    _check(load().adpsgd_state_init(C.byref(sched), C.byref(st)), "adpsgd_state_init")
+    return st
+
+
+class TraceBuffers:
+    """Host arrays for an adpsgd_trace."""
+
+    def __init__(self, cap: int):
+        import numpy as np
+        self.k = np.zeros(cap, np.int64)
+        self.p = np.zeros(cap, np.int32)
+        self.S = np.zeros(cap)
+        self.C2 = np.zeros(cap)
+        self.loss = np.zeros(cap)
+        self.phase = np.zeros(cap, np.int32)
+        self.c = Trace(cap, 0, self.k.ctypes.data_as(C.POINTER(C.c_int64)),
+                       self.p.ctypes.data_as(C.POINTER(C.c_int32)), self.S.ctypes.data_as(C.POINTER(C.c_double)),
+                       self.C2.ctypes.data_as(C.POINTER(C.c_double)),
+                       self.loss.ctypes.data_as(C.POINTER(C.c_double)),
+                       self.phase.ctypes.data_as(C.POINTER(C.c_int32)))
+
+    @property
+    def len(self) -> int:
+        return self.c.len
+
+    def arrays(self):
+        m = self.c.len
+        return dict(k=self.k[:m].copy(), p=self.p[:m].copy(), S=self.S[:m].copy(), C2=self.C2[:m].copy(),
+                    loss=self.loss[:m].copy(), phase=self.phase[:m].copy())
+
+
+def adpsgd_run(ctx: Context, sched: Schedule, state: State, k_end: int | None = None,
+               trace: TraceBuffers | None = None) -> Stats:
+    stats = Stats()
+    k_end = sched.K if k_end is None else k_end
+    _check(load().adpsgd_run(ctx.handle, C.byref(sched), C.byref(state), k_end,
+                             C.byref(trace.c) if trace is not None else None, C.byref(stats)), "adpsgd_run")
+    return stats
+
+
+def adpsgd_sched_on_sync(sched: Schedule, state: State, k: int, S: float, gamma: float) -> int:
+    ph = C.c_int32()
+    _check(load().adpsgd_sched_on_sync(C.byref(sched), C.byref(state), k, S, gamma, C.byref(ph)),
+           "adpsgd_sched_on_sync")
+    return ph.value
+
+
+def adpsgd_gamma(sched: Schedule, k: int) -> float:
+    g = C.c_float()
+    _check(load().adpsgd_gamma(C.byref(sched), k, C.byref(g)), "adpsgd_gamma")
+    return g.value
+
+
+def adpsgd_wire_bytes(n: int, P: int, rounds: int, with_scalar: bool = True):
+    pn = C.c_double()
+    tot = C.c_double()
+    _check(load().adpsgd_wire_bytes(n, P, rounds, int(with_scalar), C.byref(pn), C.byref(tot)),
+           "adpsgd_wire_bytes")
+    return pn.value, tot.value
+
+
+def adpsgd_philox_fill(seed: int, tag: int, n: int, nq: int, k: int, out, stream=None) -> None:
+    _check(load().adpsgd_philox_fill(seed & 0xFFFFFFFFFFFFFFFF, tag, n, nq, k, _ptr(out), _stream(stream)),
+           "adpsgd_philox_fill")
+
+
+def adpsgd_noise_fill_f32(seed: int, tag: int, n: int, P: int, k: int, out, stream=None) -> None:
+    _check(load().adpsgd_noise_fill_f32(seed & 0xFFFFFFFFFFFFFFFF, tag, n, P, k, _ptr(out), _stream(stream)),
+           "adpsgd_noise_fill_f32")
+
+
+def adpsgd_noise_fill_bf16(seed: int, n: int, P: int, out, stream=None) -> None:
+    _check(load().adpsgd_noise_fill_bf16(seed & 0xFFFFFFFFFFFFFFFF, n, P, _ptr(out), _stream(stream)),
+           "adpsgd_noise_fill_bf16")
+
+
+def adpsgd_kernel_times(ctx: Context):
+    a, c = C.c_double(), C.c_double()
+    b, d = C.c_int64(), C.c_int64()
+    _check(load().adpsgd_kernel_times(ctx.handle, C.byref(a), C.byref(b), C.byref(c), C.byref(d)),
+           "adpsgd_kernel_times")
+    return dict(local_step_ms=a.value, local_step_launches=b.value, average_ms=c.value,
+                average_launches=d.value)
+
+
+def adpsgd_reset_kernel_times(ctx: Context) -> None:
+    _check(load().adpsgd_reset_kernel_times(ctx.handle), "adpsgd_reset_kernel_times")
+
+
+def adpsgd_test_force_incomplete(ctx: Context, on: bool) -> None:
+    _check(load().adpsgd_test_force_incomplete(ctx.handle, int(bool(on))), "adpsgd_test_force_incomplete")
+
+
+def adpsgd_destroy(ctx: Context) -> None:
+    ctx.close()
+
+
+def adpsgd_strerror(status: int) -> str:
+    return strerror(status)
+
+
+def adpsgd_last_error() -> str:
+    return last_error()

@@ -1,0 +1,478 @@
+// kernels.cu -- sm_103a kernels of the ADPSGD hot path.
+//
+//   local_step_kernel  Algorithm 2 "updating parameter variables locally" for all n replicas in
+//                      one pass: gradient of the quadratic surrogate, Philox/Box-Muller noise
+//                      (or a pre-materialised bf16 noise tensor), weight decay, momentum and
+//                      the parameter update, 128-bit loads and stores.  HBM-bound: per
+//                      replica-param it moves x and v in and out (16 B) plus h and c once
+//                      per column (8/n B, re-reads across replicas hit L2).
+//   average_kernel     Algorithm 2 averaging + S_k: per column, the replica mean, the squared
+//                      deviations and the surrogate loss, x̄ written back to every replica;
+//                      replica values of a column stay in registers between the passes.
+//                      Persistent grid; each block leaves one fp64 partial per sum, and a
+//                      one-block kernel adds the partials in a fixed order (deterministic,
+//                      no inter-block wait).  HBM-bound: 8 B per replica-param.
+//   *_fill kernels     the raw Philox stream, its fp32 normals, and the bf16 noise tensor.
+//
+// Every fp32 operation of the update, the mean and the generator is written out once and
+// compiled with -fmad=false, so results are bit-identical to any IEEE evaluation of the same
+// sequence.
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+
+#include "launch.h"
+#include "noise.cuh"
+
+namespace adpsgd {
+
+void make_philox_keys(uint64_t seed, PhiloxKeys* out)
+{
+    uint32_t lo = (uint32_t)(seed & 0xFFFFFFFFull);
+    uint32_t hi = (uint32_t)(seed >> 32);
+    for (int r = 0; r < 10; ++r) {
+        out->lo[r] = lo;
+        out->hi[r] = hi;
+        lo += 0x9E3779B9u;  // Weyl constants of Philox4x32
+        hi += 0xBB67AE85u;
+    }
+}
+
+namespace {
+
+constexpr int kThreads = 256;
+
+// ------------------------------------------------------------------------------------------
+// Local step
+// ------------------------------------------------------------------------------------------
+struct StepParams {
+    float* x;
+    float* v;
+    const float* h;
+    const float* c;
+    const uint16_t* noise;
+    int64_t P;
+    int64_t Q;  // ceil(P / 4): blocks of four elements, one Philox call each
+    int32_t n;
+    uint32_t k;
+    float gamma, mu, wd, sigma;
+    PhiloxKeys keys;
+};
+
+// g = h (x - c) + sigma z [+ wd x];  v = mu v + g;  x = x - gamma v  (one rounding each).
+template <bool WD>
+__device__ __forceinline__ void sgd_update(float& x, float& v, float h, float c, float z,
+                                           float gamma, float mu, float wd, float sigma)
+{
+    const float diff = x - c;
+    float g = h * diff;
+    const float noise = sigma * z;
+    g = g + noise;
+    if (WD) {
+        const float decay = wd * x;
+        g = g + decay;
+    }
+    const float mv = mu * v;
+    const float vnew = mv + g;
+    const float step = gamma * vnew;
+    v = vnew;
+    x = x - step;
+}
+
+__device__ __forceinline__ float bf16_bits_to_float(uint32_t bits16) { return __uint_as_float(bits16 << 16); }
+
+// Block b handles replica i = b mod n and blocks of four columns q = (b div n) * 256 + tid, so
+// the n blocks that read the same h, c tile run back to back (the re-reads hit L2).
+template <bool VEC, bool BF16, bool WD>
+__global__ void __launch_bounds__(kThreads) local_step_kernel(const StepParams p)
+{
+    const int64_t b = blockIdx.x;
+    const int32_t i = (int32_t)(b % p.n);
+    const int64_t q = (b / p.n) * kThreads + threadIdx.x;
+    if (q >= p.Q) return;
+    const int64_t row = (int64_t)i * p.P;
+    if (VEC) {
+        float4* __restrict__ xp = reinterpret_cast<float4*>(p.x + row) + q;
+        float4* __restrict__ vp = reinterpret_cast<float4*>(p.v + row) + q;
+        float4 xv = *xp;
+        float4 vv = *vp;
+        const float4 hv = __ldg(reinterpret_cast<const float4*>(p.h) + q);
+        const float4 cv = __ldg(reinterpret_cast<const float4*>(p.c) + q);
+        float4 z;
+        if (BF16) {
+            const uint2 nb = __ldg(reinterpret_cast<const uint2*>(p.noise + row) + q);
+            z = make_float4(bf16_bits_to_float(nb.x & 0xFFFFu), __uint_as_float(nb.x & 0xFFFF0000u),
+                            bf16_bits_to_float(nb.y & 0xFFFFu), __uint_as_float(nb.y & 0xFFFF0000u));
+        } else {
+            z = normals4(p.keys, (uint32_t)q, (uint32_t)i, p.k, 0u);
+        }
+        sgd_update<WD>(xv.x, vv.x, hv.x, cv.x, z.x, p.gamma, p.mu, p.wd, p.sigma);
+        sgd_update<WD>(xv.y, vv.y, hv.y, cv.y, z.y, p.gamma, p.mu, p.wd, p.sigma);
+        sgd_update<WD>(xv.z, vv.z, hv.z, cv.z, z.z, p.gamma, p.mu, p.wd, p.sigma);
+        sgd_update<WD>(xv.w, vv.w, hv.w, cv.w, z.w, p.gamma, p.mu, p.wd, p.sigma);
+        *xp = xv;
+        *vp = vv;
+    } else {
+        float zz[4];
+        if (!BF16) {
+            const float4 z = normals4(p.keys, (uint32_t)q, (uint32_t)i, p.k, 0u);
+            zz[0] = z.x; zz[1] = z.y; zz[2] = z.z; zz[3] = z.w;
+        }
+#pragma unroll
+        for (int r = 0; r < 4; ++r) {
+            const int64_t j = 4 * q + r;
+            if (j >= p.P) break;
+            float xs = p.x[row + j];
+            float vs = p.v[row + j];
+            const float z = BF16 ? bf16_bits_to_float(p.noise[row + j]) : zz[r];
+            sgd_update<WD>(xs, vs, __ldg(p.h + j), __ldg(p.c + j), z, p.gamma, p.mu, p.wd, p.sigma);
+            p.x[row + j] = xs;
+            p.v[row + j] = vs;
+        }
+    }
+}
+
+// ------------------------------------------------------------------------------------------
+// Averaging + variance
+// ------------------------------------------------------------------------------------------
+struct AvgParams {
+    float* x;
+    const float* h;
+    const float* c;
+    int64_t P;
+    int64_t Q;  // columns (scalar) or blocks of four columns (vector) handled by one thread
+    int32_t n;
+    double* partials;
+};
+
+// Fixed-order block sum; the result is valid in thread 0.
+__device__ __forceinline__ double block_sum(double v, double* shared)
+{
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) v += __shfl_down_sync(0xFFFFFFFFu, v, off);
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    if (lane == 0) shared[warp] = v;
+    __syncthreads();
+    double total = 0.0;
+    if (threadIdx.x == 0)
+        for (int w = 0; w < kThreads / 32; ++w) total += shared[w];
+    __syncthreads();
+    return total;
+}
+
+// Per-column statistics of one column held as values r_0 .. r_{n-1}:
+// xbar = r_0 + (sum_{i>=1} (r_i - r_0)) / n   and   d = sum_i (r_i - xbar)^2  (fp32).
+template <int NMAX>
+__device__ __forceinline__ void column_stats(const float* r, int n, float nf, float& xbar, float& d)
+{
+    const float base = r[0];
+    float acc = 0.0f;
+#pragma unroll
+    for (int i = 1; i < NMAX; ++i)
+        if (i < n) acc = acc + (r[i] - base);
+    xbar = base + __fdiv_rn(acc, nf);
+    float s = 0.0f;
+#pragma unroll
+    for (int i = 0; i < NMAX; ++i)
+        if (i < n) {
+            const float dev = r[i] - xbar;
+            s = s + dev * dev;
+        }
+    d = s;
+}
+
+// Columns with more than 32 replicas: the same arithmetic, re-reading x (L1/L2) per pass.
+__device__ __forceinline__ void column_stats_global(const float* x, int64_t P, int64_t j, int n, float nf,
+                                                    float& xbar, float& d)
+{
+    const float base = x[j];
+    float acc = 0.0f;
+    for (int i = 1; i < n; ++i) acc = acc + (x[(int64_t)i * P + j] - base);
+    xbar = base + __fdiv_rn(acc, nf);
+    float s = 0.0f;
+    for (int i = 0; i < n; ++i) {
+        const float dev = x[(int64_t)i * P + j] - xbar;
+        s = s + dev * dev;
+    }
+    d = s;
+}
+
+template <int NMAX, bool VEC, bool LOSS, bool WRITE>
+__global__ void __launch_bounds__(kThreads) average_kernel(const AvgParams p)
+{
+    __shared__ double shared[kThreads / 32];
+    const int32_t n = p.n;
+    const float nf = (float)n;
+    double accD = 0.0, accL = 0.0;
+    const int64_t stride = (int64_t)gridDim.x * kThreads;
+    for (int64_t q = (int64_t)blockIdx.x * kThreads + threadIdx.x; q < p.Q; q += stride) {
+        if (VEC) {
+            float xbar[4], d[4];
+            if (NMAX > 0) {
+                constexpr int R = NMAX > 0 ? NMAX : 1;
+                float4 r4[R];
+#pragma unroll
+                for (int i = 0; i < R; ++i)
+                    if (i < n) r4[i] = reinterpret_cast<const float4*>(p.x + (int64_t)i * p.P)[q];
+                float col[R];
+#pragma unroll
+                for (int i = 0; i < R; ++i) col[i] = (i < n) ? r4[i].x : 0.0f;
+                column_stats<R>(col, n, nf, xbar[0], d[0]);
+#pragma unroll
+                for (int i = 0; i < R; ++i) col[i] = (i < n) ? r4[i].y : 0.0f;
+                column_stats<R>(col, n, nf, xbar[1], d[1]);
+#pragma unroll
+                for (int i = 0; i < R; ++i) col[i] = (i < n) ? r4[i].z : 0.0f;
+                column_stats<R>(col, n, nf, xbar[2], d[2]);
+#pragma unroll
+                for (int i = 0; i < R; ++i) col[i] = (i < n) ? r4[i].w : 0.0f;
+                column_stats<R>(col, n, nf, xbar[3], d[3]);
+            } else {
+#pragma unroll
+                for (int r = 0; r < 4; ++r) column_stats_global(p.x, p.P, 4 * q + r, n, nf, xbar[r], d[r]);
+            }
+            accD += (double)((d[0] + d[1]) + (d[2] + d[3]));
+            if (LOSS) {
+                const float4 hv = __ldg(reinterpret_cast<const float4*>(p.h) + q);
+                const float4 cv = __ldg(reinterpret_cast<const float4*>(p.c) + q);
+                const float t0 = xbar[0] - cv.x, t1 = xbar[1] - cv.y, t2 = xbar[2] - cv.z, t3 = xbar[3] - cv.w;
+                const float l0 = (hv.x * t0) * t0, l1 = (hv.y * t1) * t1;
+                const float l2 = (hv.z * t2) * t2, l3 = (hv.w * t3) * t3;
+                accL += (double)((l0 + l1) + (l2 + l3));
+            }
+            if (WRITE) {
+                const float4 out = make_float4(xbar[0], xbar[1], xbar[2], xbar[3]);
+                for (int i = 0; i < n; ++i) reinterpret_cast<float4*>(p.x + (int64_t)i * p.P)[q] = out;
+            }
+        } else {
+            const int64_t j = q;
+            float xbar, d;
+            if (NMAX > 0) {
+                constexpr int R = NMAX > 0 ? NMAX : 1;
+                float col[R];
+#pragma unroll
+                for (int i = 0; i < R; ++i) col[i] = (i < n) ? p.x[(int64_t)i * p.P + j] : 0.0f;
+                column_stats<R>(col, n, nf, xbar, d);
+            } else {
+                column_stats_global(p.x, p.P, j, n, nf, xbar, d);
+            }
+            accD += (double)d;
+            if (LOSS) {
+                const float t = xbar - __ldg(p.c + j);
+                const float l = (__ldg(p.h + j) * t) * t;
+                accL += (double)l;
+            }
+            if (WRITE)
+                for (int i = 0; i < n; ++i) p.x[(int64_t)i * p.P + j] = xbar;
+        }
+    }
+    const double bD = block_sum(accD, shared);
+    const double bL = LOSS ? block_sum(accL, shared) : 0.0;
+    if (threadIdx.x == 0) {
+        p.partials[blockIdx.x] = bD;
+        p.partials[gridDim.x + blockIdx.x] = bL;
+    }
+}
+
+// out[0] = sum of the D partials, out[1] = 1/2 sum of the loss partials, in a fixed order.
+__global__ void __launch_bounds__(kThreads) finalize_kernel(const double* partials, int nblocks, double* out)
+{
+    __shared__ double shared[kThreads / 32];
+    double d = 0.0, l = 0.0;
+    for (int b = threadIdx.x; b < nblocks; b += kThreads) {
+        d += partials[b];
+        l += partials[nblocks + b];
+    }
+    d = block_sum(d, shared);
+    l = block_sum(l, shared);
+    if (threadIdx.x == 0) {
+        out[0] = d;
+        out[1] = 0.5 * l;
+    }
+}
+
+// ------------------------------------------------------------------------------------------
+// Generator fills
+// ------------------------------------------------------------------------------------------
+__global__ void __launch_bounds__(kThreads) philox_fill_kernel(PhiloxKeys keys, uint32_t tag, int32_t n,
+                                                               int64_t nq, uint32_t k, uint4* out)
+{
+    const int64_t t = (int64_t)blockIdx.x * kThreads + threadIdx.x;
+    if (t >= (int64_t)n * nq) return;
+    const uint32_t i = (uint32_t)(t / nq);
+    const uint32_t q = (uint32_t)(t % nq);
+    out[t] = philox4x32_10(make_uint4(q, i, k, tag), keys);
+}
+
+__global__ void __launch_bounds__(kThreads) noise_f32_kernel(PhiloxKeys keys, uint32_t tag, int32_t n,
+                                                             int64_t P, int64_t Q, uint32_t k, float* out)
+{
+    const int64_t t = (int64_t)blockIdx.x * kThreads + threadIdx.x;
+    if (t >= (int64_t)n * Q) return;
+    const int64_t i = t / Q, q = t % Q;
+    const float4 z = normals4(keys, (uint32_t)q, (uint32_t)i, k, tag);
+    const float zz[4] = {z.x, z.y, z.z, z.w};
+#pragma unroll
+    for (int r = 0; r < 4; ++r)
+        if (4 * q + r < P) out[i * P + 4 * q + r] = zz[r];
+}
+
+__global__ void __launch_bounds__(kThreads) noise_bf16_kernel(PhiloxKeys keys, int32_t n, int64_t P,
+                                                              int64_t Q, uint16_t* out)
+{
+    const int64_t t = (int64_t)blockIdx.x * kThreads + threadIdx.x;
+    if (t >= (int64_t)n * Q) return;
+    const int64_t i = t / Q, q = t % Q;
+    const float4 z = normals4(keys, (uint32_t)q, (uint32_t)i, 0u, 1u);
+    const float zz[4] = {z.x, z.y, z.z, z.w};
+#pragma unroll
+    for (int r = 0; r < 4; ++r)
+        if (4 * q + r < P) out[i * P + 4 * q + r] = __bfloat16_as_ushort(__float2bfloat16_rn(zz[r]));
+}
+
+template <typename Kernel>
+int max_blocks_per_sm(Kernel kernel)
+{
+    int nb = 0;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&nb, kernel, kThreads, 0) != cudaSuccess) {
+        cudaGetLastError();
+        nb = 1;
+    }
+    return nb < 1 ? 1 : nb;
+}
+
+using AvgKernel = void (*)(const AvgParams);
+
+template <int NMAX>
+AvgKernel pick_average_nmax(bool vec, bool loss, bool write)
+{
+    if (vec) {
+        if (!write) return average_kernel<NMAX, true, false, false>;
+        return loss ? average_kernel<NMAX, true, true, true> : average_kernel<NMAX, true, false, true>;
+    }
+    if (!write) return average_kernel<NMAX, false, false, false>;
+    return loss ? average_kernel<NMAX, false, true, true> : average_kernel<NMAX, false, false, true>;
+}
+
+AvgKernel pick_average(int32_t n, bool vec, bool loss, bool write)
+{
+    if (n <= 4) return pick_average_nmax<4>(vec, loss, write);
+    if (n <= 8) return pick_average_nmax<8>(vec, loss, write);
+    if (n <= 16) return pick_average_nmax<16>(vec, loss, write);
+    if (n <= 32) return pick_average_nmax<32>(vec, loss, write);
+    return pick_average_nmax<0>(vec, loss, write);
+}
+
+bool use_vec(int64_t P, const void* a, const void* b, const void* c, const void* d)
+{
+    auto al = [](const void* ptr) { return ptr == nullptr || (reinterpret_cast<uintptr_t>(ptr) & 15u) == 0; };
+    return (P % 4 == 0) && al(a) && al(b) && al(c) && al(d);
+}
+
+int64_t ceil_div(int64_t a, int64_t b) { return (a + b - 1) / b; }
+
+}  // namespace
+
+cudaError_t launch_local_step(const LocalStepArgs& a, cudaStream_t stream)
+{
+    StepParams p;
+    p.x = a.x;
+    p.v = a.v;
+    p.h = a.h;
+    p.c = a.c;
+    p.noise = a.noise_bf16;
+    p.P = a.P;
+    p.Q = ceil_div(a.P, 4);
+    p.n = a.n;
+    p.k = a.k;
+    p.gamma = a.gamma;
+    p.mu = a.mu;
+    p.wd = a.wd;
+    p.sigma = a.sigma;
+    p.keys = *a.keys;
+    const bool vec = use_vec(a.P, a.x, a.v, a.h, a.c) &&
+                     (a.noise_bf16 == nullptr || (reinterpret_cast<uintptr_t>(a.noise_bf16) & 7u) == 0);
+    const bool bf16 = a.noise_bf16 != nullptr;
+    const bool wd = a.wd != 0.0f;
+    const int64_t blocks = (int64_t)a.n * ceil_div(p.Q, kThreads);
+    void (*kernel)(const StepParams);
+    if (vec) {
+        if (bf16) kernel = wd ? local_step_kernel<true, true, true> : local_step_kernel<true, true, false>;
+        else kernel = wd ? local_step_kernel<true, false, true> : local_step_kernel<true, false, false>;
+    } else {
+        if (bf16) kernel = wd ? local_step_kernel<false, true, true> : local_step_kernel<false, true, false>;
+        else kernel = wd ? local_step_kernel<false, false, true> : local_step_kernel<false, false, false>;
+    }
+    kernel<<<(unsigned)blocks, kThreads, 0, stream>>>(p);
+    return cudaGetLastError();
+}
+
+int average_grid_max(int sms) { return sms * (2048 / kThreads); }
+
+int average_grid(int32_t n, int64_t P, bool loss, bool write_back, int sms)
+{
+    // vector-ness does not change the occupancy enough to matter; size for the vector kernel
+    const AvgKernel kernel = pick_average(n, true, loss, write_back);
+    const int per_sm = max_blocks_per_sm(kernel);
+    const int64_t work = ceil_div(ceil_div(P, 4), kThreads);
+    int64_t grid = (int64_t)per_sm * sms;
+    if (grid > work) grid = work;
+    if (grid < 1) grid = 1;
+    const int cap = average_grid_max(sms);
+    return (int)(grid > cap ? cap : grid);
+}
+
+cudaError_t launch_average(const AverageArgs& a, cudaStream_t stream)
+{
+    const bool loss = a.h != nullptr;
+    const bool vec = use_vec(a.P, a.x, a.h, a.c, nullptr);
+    AvgParams p;
+    p.x = a.x;
+    p.h = a.h;
+    p.c = a.c;
+    p.P = a.P;
+    p.Q = vec ? a.P / 4 : a.P;
+    p.n = a.n;
+    p.partials = a.partials;
+    const AvgKernel kernel = pick_average(a.n, vec, loss, a.write_back);
+    kernel<<<a.grid, kThreads, 0, stream>>>(p);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    finalize_kernel<<<1, kThreads, 0, stream>>>(a.partials, a.grid, a.out);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_philox_fill(uint64_t seed, uint32_t tag, int32_t n, int64_t nq, uint32_t k,
+                               uint32_t* out, cudaStream_t stream)
+{
+    PhiloxKeys keys;
+    make_philox_keys(seed, &keys);
+    const int64_t blocks = ceil_div((int64_t)n * nq, kThreads);
+    if (blocks == 0) return cudaSuccess;
+    philox_fill_kernel<<<(unsigned)blocks, kThreads, 0, stream>>>(keys, tag, n, nq, k, reinterpret_cast<uint4*>(out));
+    return cudaGetLastError();
+}
+
+cudaError_t launch_noise_f32(uint64_t seed, uint32_t tag, int32_t n, int64_t P, uint32_t k, float* out,
+                             cudaStream_t stream)
+{
+    PhiloxKeys keys;
+    make_philox_keys(seed, &keys);
+    const int64_t Q = ceil_div(P, 4);
+    const int64_t blocks = ceil_div((int64_t)n * Q, kThreads);
+    if (blocks == 0) return cudaSuccess;
+    noise_f32_kernel<<<(unsigned)blocks, kThreads, 0, stream>>>(keys, tag, n, P, Q, k, out);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_noise_bf16(uint64_t seed, int32_t n, int64_t P, uint16_t* out, cudaStream_t stream)
+{
+    PhiloxKeys keys;
+    make_philox_keys(seed, &keys);
+    const int64_t Q = ceil_div(P, 4);
+    const int64_t blocks = ceil_div((int64_t)n * Q, kThreads);
+    if (blocks == 0) return cudaSuccess;
+    noise_bf16_kernel<<<(unsigned)blocks, kThreads, 0, stream>>>(keys, n, P, Q, out);
+    return cudaGetLastError();
+}
+
+}  // namespace adpsgd

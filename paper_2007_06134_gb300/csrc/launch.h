@@ -1,0 +1,60 @@
+// launch.h -- internal interface between the host runtime and the CUDA kernels.
+#pragma once
+
+#include <cuda_runtime_api.h>
+
+#include <cstdint>
+
+namespace adpsgd {
+
+// Round keys of Philox4x32-10 for one seed: key r = key 0 + r * (Weyl constants).
+struct PhiloxKeys {
+    uint32_t lo[10];
+    uint32_t hi[10];
+};
+
+// Round keys of Philox4x32-10 for a 64-bit seed (key = (seed lo, seed hi), bumped by the
+// Weyl constants once per round).
+void make_philox_keys(uint64_t seed, PhiloxKeys* out);
+
+// One local step of every replica (Algorithm 2, update line).
+struct LocalStepArgs {
+    float* x;
+    float* v;
+    const float* h;
+    const float* c;
+    const uint16_t* noise_bf16;  // nullptr: Philox noise
+    const PhiloxKeys* keys;
+    int32_t n;
+    int64_t P;
+    uint32_t k;
+    float gamma, mu, wd, sigma;
+};
+cudaError_t launch_local_step(const LocalStepArgs& a, cudaStream_t stream);
+
+// Averaging + variance (+ loss): per-block fp64 partials, then a one-block fixed-order sum
+// into out[0] (D) and out[1] (loss).
+struct AverageArgs {
+    float* x;
+    const float* h;  // nullptr unless the loss is wanted
+    const float* c;
+    int32_t n;
+    int64_t P;
+    bool write_back;  // false: variance only
+    double* partials; // 2 * grid doubles
+    double* out;      // 2 doubles
+    int grid;         // from average_grid()
+};
+cudaError_t launch_average(const AverageArgs& a, cudaStream_t stream);
+// Blocks of the persistent averaging kernel for this shape on a device with `sms` SMs.
+int average_grid(int32_t n, int64_t P, bool loss, bool write_back, int sms);
+int average_grid_max(int sms);
+
+cudaError_t launch_philox_fill(uint64_t seed, uint32_t tag, int32_t n, int64_t nq, uint32_t k,
+                               uint32_t* out, cudaStream_t stream);
+cudaError_t launch_noise_f32(uint64_t seed, uint32_t tag, int32_t n, int64_t P, uint32_t k,
+                             float* out, cudaStream_t stream);
+cudaError_t launch_noise_bf16(uint64_t seed, int32_t n, int64_t P, uint16_t* out,
+                              cudaStream_t stream);
+
+}  // namespace adpsgd

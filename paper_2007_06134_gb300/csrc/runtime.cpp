@@ -1,0 +1,519 @@
+// runtime.cpp -- host side of the C ABI in include/adpsgd.h: argument checks, the context,
+// the ADPSGD period rule (Algorithm 2), the step-size schedule, the run loop and the bounded
+// waits.  All device work goes through the kernels in kernels.cu on the caller's stream.
+#include <cuda_runtime_api.h>
+
+#include <chrono>
+#include <cstdint>
+#include <cstdio>
+#include <cstring>
+#include <new>
+#include <string>
+#include <thread>
+#include <vector>
+
+#include "../../include/adpsgd.h"
+#include "launch.h"
+
+namespace {
+
+thread_local std::string g_last_error;
+
+int cuda_fail(cudaError_t e, const char* where)
+{
+    g_last_error = std::string(where) + ": " + cudaGetErrorName(e) + ": " + cudaGetErrorString(e);
+    return ADPSGD_E_CUDA;
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+constexpr int64_t kMaxK = int64_t(1) << 32;  // the step index is one 32-bit Philox counter word
+
+}  // namespace
+
+struct TimedLaunch {
+    cudaEvent_t start, stop;
+    int kind;  // 0 local step, 1 averaging
+};
+
+struct adpsgd_ctx {
+    adpsgd_config cfg{};
+    float* x = nullptr;
+    float* v = nullptr;
+    const float* h = nullptr;
+    const float* c = nullptr;
+    const uint16_t* noise = nullptr;
+    cudaStream_t stream = nullptr;
+    int device = 0;
+    int sms = 0;
+    adpsgd::PhiloxKeys keys{};
+    double* d_partials = nullptr;
+    double* d_out = nullptr;
+    double* h_out = nullptr;  // pinned, 2 doubles
+    cudaEvent_t done = nullptr;
+    int grid_avg = 0, grid_avg_loss = 0, grid_var = 0;
+    // kernel timing
+    std::vector<cudaEvent_t> free_events;
+    std::vector<TimedLaunch> pending;
+    double ms[2] = {0.0, 0.0};
+    int64_t launches[2] = {0, 0};
+    int64_t timed_launches[2] = {0, 0};
+    bool force_incomplete = false;
+};
+
+namespace {
+
+int64_t timeout_ms(const adpsgd_ctx* ctx)
+{
+    return ctx->cfg.wait_timeout_ms > 0 ? ctx->cfg.wait_timeout_ms : 60000;
+}
+
+// Poll an event until it completes or the context's time limit passes.
+int wait_event(adpsgd_ctx* ctx, cudaEvent_t ev)
+{
+    const auto t0 = std::chrono::steady_clock::now();
+    const auto limit = std::chrono::milliseconds(timeout_ms(ctx));
+    int spins = 0;
+    for (;;) {
+        cudaError_t e = ctx->force_incomplete ? cudaErrorNotReady : cudaEventQuery(ev);
+        if (e == cudaSuccess) return ADPSGD_OK;
+        if (e != cudaErrorNotReady) return cuda_fail(e, "cudaEventQuery");
+        if (std::chrono::steady_clock::now() - t0 > limit) {
+            g_last_error = "bounded wait ran out";
+            return ADPSGD_E_TIMEOUT;
+        }
+        if (++spins > 2000) std::this_thread::sleep_for(std::chrono::microseconds(20));
+    }
+}
+
+int take_event(adpsgd_ctx* ctx, cudaEvent_t* ev)
+{
+    if (!ctx->free_events.empty()) {
+        *ev = ctx->free_events.back();
+        ctx->free_events.pop_back();
+        return ADPSGD_OK;
+    }
+    cudaError_t e = cudaEventCreate(ev);
+    return e == cudaSuccess ? ADPSGD_OK : cuda_fail(e, "cudaEventCreate");
+}
+
+// Add up the elapsed times of all recorded launches (all of them must have completed).
+int harvest_times(adpsgd_ctx* ctx)
+{
+    if (ctx->pending.empty()) return ADPSGD_OK;
+    int st = wait_event(ctx, ctx->pending.back().stop);
+    if (st != ADPSGD_OK) return st;
+    for (const TimedLaunch& t : ctx->pending) {
+        float ms = 0.0f;
+        cudaError_t e = cudaEventElapsedTime(&ms, t.start, t.stop);
+        if (e != cudaSuccess) return cuda_fail(e, "cudaEventElapsedTime");
+        ctx->ms[t.kind] += ms;
+        ctx->timed_launches[t.kind] += 1;
+        ctx->free_events.push_back(t.start);
+        ctx->free_events.push_back(t.stop);
+    }
+    ctx->pending.clear();
+    return ADPSGD_OK;
+}
+
+template <typename Launch>
+int timed(adpsgd_ctx* ctx, int kind, Launch launch, const char* what)
+{
+    cudaEvent_t a = nullptr, b = nullptr;
+    if (ctx->cfg.time_kernels) {
+        if (ctx->pending.size() >= 4096) {
+            int st = harvest_times(ctx);
+            if (st != ADPSGD_OK) return st;
+        }
+        int st = take_event(ctx, &a);
+        if (st == ADPSGD_OK) st = take_event(ctx, &b);
+        if (st != ADPSGD_OK) return st;
+        cudaError_t e = cudaEventRecord(a, ctx->stream);
+        if (e != cudaSuccess) return cuda_fail(e, "cudaEventRecord");
+    }
+    cudaError_t e = launch();
+    if (e != cudaSuccess) return cuda_fail(e, what);
+    ctx->launches[kind] += 1;
+    if (ctx->cfg.time_kernels) {
+        e = cudaEventRecord(b, ctx->stream);
+        if (e != cudaSuccess) return cuda_fail(e, "cudaEventRecord");
+        ctx->pending.push_back({a, b, kind});
+    }
+    return ADPSGD_OK;
+}
+
+int local_step(adpsgd_ctx* ctx, int64_t k, float gamma)
+{
+    adpsgd::LocalStepArgs a;
+    a.x = ctx->x;
+    a.v = ctx->v;
+    a.h = ctx->h;
+    a.c = ctx->c;
+    a.noise_bf16 = ctx->cfg.noise_mode == ADPSGD_NOISE_BF16 ? ctx->noise : nullptr;
+    a.keys = &ctx->keys;
+    a.n = ctx->cfg.n;
+    a.P = ctx->cfg.P;
+    a.k = (uint32_t)k;
+    a.gamma = gamma;
+    a.mu = ctx->cfg.momentum;
+    a.wd = ctx->cfg.weight_decay;
+    a.sigma = ctx->cfg.noise_sigma;
+    return timed(ctx, 0, [&] { return adpsgd::launch_local_step(a, ctx->stream); }, "local step");
+}
+
+// Averaging (write_back) or variance only; results land in ctx->h_out after a bounded wait.
+int average(adpsgd_ctx* ctx, bool write_back, bool loss)
+{
+    adpsgd::AverageArgs a;
+    a.x = ctx->x;
+    a.h = loss ? ctx->h : nullptr;
+    a.c = loss ? ctx->c : nullptr;
+    a.n = ctx->cfg.n;
+    a.P = ctx->cfg.P;
+    a.write_back = write_back;
+    a.partials = ctx->d_partials;
+    a.out = ctx->d_out;
+    a.grid = !write_back ? ctx->grid_var : (loss ? ctx->grid_avg_loss : ctx->grid_avg);
+    int st = timed(ctx, 1, [&] { return adpsgd::launch_average(a, ctx->stream); }, "average");
+    if (st != ADPSGD_OK) return st;
+    cudaError_t e = cudaMemcpyAsync(ctx->h_out, ctx->d_out, 2 * sizeof(double), cudaMemcpyDeviceToHost,
+                                    ctx->stream);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaMemcpyAsync");
+    e = cudaEventRecord(ctx->done, ctx->stream);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaEventRecord");
+    st = wait_event(ctx, ctx->done);
+    if (st != ADPSGD_OK) return st;
+    if (ctx->cfg.time_kernels) return harvest_times(ctx);
+    return ADPSGD_OK;
+}
+
+int check_schedule(const adpsgd_schedule* s)
+{
+    if (s == nullptr) return ADPSGD_E_INVAL;
+    if (s->kind != ADPSGD_CPSGD && s->kind != ADPSGD_ADPSGD) return ADPSGD_E_INVAL;
+    if (s->p_init < 1 || s->K < 0 || s->K > kMaxK || s->K_w < 0 || s->K_s < 0) return ADPSGD_E_INVAL;
+    if (s->p_min < 1 || s->p_max < 0 || (s->p_max > 0 && s->p_max < s->p_min)) return ADPSGD_E_INVAL;
+    if (s->n_milestones < 0 || (s->n_milestones > 0 && s->milestones == nullptr)) return ADPSGD_E_INVAL;
+    if (!(s->lr0 > 0.0) || !(s->lr_factor > 0.0)) return ADPSGD_E_INVAL;
+    if (s->kind == ADPSGD_ADPSGD) {
+        if (s->literal_phase) return ADPSGD_E_INVAL;
+        if (!(s->lo > 0.0) || !(s->hi >= s->lo)) return ADPSGD_E_INVAL;
+        // C_2 must receive at least one sample before the rule first compares against it.
+        if (s->K_s < s->K_w + s->p_init) return ADPSGD_E_INVAL;
+    }
+    return ADPSGD_OK;
+}
+
+float gamma_of(const adpsgd_schedule* s, int64_t k)
+{
+    double g = s->lr0;
+    for (int32_t t = 0; t < s->n_milestones; ++t)
+        if (k >= s->milestones[t]) g = g * s->lr_factor;
+    return (float)g;
+}
+
+// Does iteration k end with a sync?  Advances cnt like Algorithm 2.
+bool sync_after(const adpsgd_schedule* s, adpsgd_state* st, int64_t k)
+{
+    if (k < s->K_w) {
+        st->cnt = 0;
+        return true;
+    }
+    if (s->kind == ADPSGD_CPSGD && s->literal_phase) return (k % st->p) == 0;
+    st->cnt += 1;
+    if (st->cnt >= st->p) {
+        st->cnt = 0;
+        return true;
+    }
+    return false;
+}
+
+int32_t rule(const adpsgd_schedule* s, adpsgd_state* st, int64_t k, double S, double gamma)
+{
+    if (k < s->K_w) return 1;                 // warm-up
+    if (s->kind == ADPSGD_CPSGD) return 0;    // constant period
+    if (k < s->K_s) {                         // sampling C_2 (cumulative mean)
+        st->m += 1;
+        st->C2 += (S / gamma - st->C2) / (double)st->m;
+        return 2;
+    }
+    const double target = gamma * st->C2;
+    if (S < s->lo * target) st->p += 1;
+    else if (S > s->hi * target) st->p -= 1;
+    if (st->p < s->p_min) st->p = s->p_min;
+    if (s->p_max > 0 && st->p > s->p_max) st->p = s->p_max;
+    return 3;
+}
+
+void wire(int32_t n, int64_t P, int64_t rounds, bool with_scalar, double* per_node, double* total)
+{
+    const double ring = 2.0 * (double)(n - 1) / (double)n;
+    double per_round = ring * 4.0 * (double)P;
+    if (with_scalar) per_round += ring * 4.0;
+    *per_node = per_round * (double)rounds;
+    *total = *per_node * (double)n;
+}
+
+}  // namespace
+
+extern "C" {
+
+const char* adpsgd_strerror(int status)
+{
+    switch (status) {
+    case ADPSGD_OK: return "ok";
+    case ADPSGD_E_INVAL: return "invalid argument";
+    case ADPSGD_E_ALIGN: return "device pointer not 16-byte aligned";
+    case ADPSGD_E_CUDA: return "CUDA error";
+    case ADPSGD_E_TIMEOUT: return "bounded wait timed out";
+    case ADPSGD_E_NOMEM: return "out of memory";
+    case ADPSGD_E_STATE: return "invalid state for this call";
+    default: return "unknown status";
+    }
+}
+
+const char* adpsgd_last_error(void) { return g_last_error.c_str(); }
+
+int adpsgd_init(const adpsgd_config* cfg, float* x, float* v, const float* h, const float* c,
+                const uint16_t* noise_bf16, void* stream, adpsgd_ctx** out)
+{
+    if (out == nullptr) return ADPSGD_E_INVAL;
+    *out = nullptr;
+    if (cfg == nullptr || x == nullptr || v == nullptr || h == nullptr || c == nullptr) return ADPSGD_E_INVAL;
+    if (cfg->n < 1 || cfg->P < 1) return ADPSGD_E_INVAL;
+    if (cfg->P > (int64_t(1) << 34) || (int64_t)cfg->n * cfg->P > (int64_t(1) << 40)) return ADPSGD_E_INVAL;
+    if (cfg->noise_mode != ADPSGD_NOISE_PHILOX && cfg->noise_mode != ADPSGD_NOISE_BF16) return ADPSGD_E_INVAL;
+    if (cfg->noise_mode == ADPSGD_NOISE_BF16 && noise_bf16 == nullptr) return ADPSGD_E_INVAL;
+    if (!aligned16(x) || !aligned16(v) || !aligned16(h) || !aligned16(c)) return ADPSGD_E_ALIGN;
+    if (noise_bf16 != nullptr && !aligned16(noise_bf16)) return ADPSGD_E_ALIGN;
+
+    adpsgd_ctx* ctx = new (std::nothrow) adpsgd_ctx();
+    if (ctx == nullptr) return ADPSGD_E_NOMEM;
+    ctx->cfg = *cfg;
+    ctx->x = x;
+    ctx->v = v;
+    ctx->h = h;
+    ctx->c = c;
+    ctx->noise = cfg->noise_mode == ADPSGD_NOISE_BF16 ? noise_bf16 : nullptr;
+    ctx->stream = static_cast<cudaStream_t>(stream);
+    adpsgd::make_philox_keys(cfg->seed, &ctx->keys);
+
+    cudaError_t e = cudaGetDevice(&ctx->device);
+    if (e == cudaSuccess) e = cudaDeviceGetAttribute(&ctx->sms, cudaDevAttrMultiProcessorCount, ctx->device);
+    if (e != cudaSuccess) {
+        delete ctx;
+        return cuda_fail(e, "device query");
+    }
+    ctx->grid_avg = adpsgd::average_grid(cfg->n, cfg->P, false, true, ctx->sms);
+    ctx->grid_avg_loss = adpsgd::average_grid(cfg->n, cfg->P, true, true, ctx->sms);
+    ctx->grid_var = adpsgd::average_grid(cfg->n, cfg->P, false, false, ctx->sms);
+    const size_t partial_bytes = 2 * sizeof(double) * (size_t)adpsgd::average_grid_max(ctx->sms);
+    e = cudaMalloc(reinterpret_cast<void**>(&ctx->d_partials), partial_bytes);
+    if (e == cudaSuccess) e = cudaMalloc(reinterpret_cast<void**>(&ctx->d_out), 2 * sizeof(double));
+    if (e == cudaSuccess) e = cudaMallocHost(reinterpret_cast<void**>(&ctx->h_out), 2 * sizeof(double));
+    if (e == cudaSuccess) e = cudaEventCreateWithFlags(&ctx->done, cudaEventDisableTiming);
+    if (e != cudaSuccess) {
+        adpsgd_destroy(ctx);
+        cudaGetLastError();
+        g_last_error = std::string("context allocation: ") + cudaGetErrorString(e);
+        return e == cudaErrorMemoryAllocation ? ADPSGD_E_NOMEM : ADPSGD_E_CUDA;
+    }
+    *out = ctx;
+    return ADPSGD_OK;
+}
+
+void adpsgd_destroy(adpsgd_ctx* ctx)
+{
+    if (ctx == nullptr) return;
+    if (ctx->done != nullptr && cudaEventRecord(ctx->done, ctx->stream) == cudaSuccess) {
+        bool forced = ctx->force_incomplete;
+        ctx->force_incomplete = false;
+        wait_event(ctx, ctx->done);
+        ctx->force_incomplete = forced;
+    }
+    for (const TimedLaunch& t : ctx->pending) {
+        cudaEventDestroy(t.start);
+        cudaEventDestroy(t.stop);
+    }
+    for (cudaEvent_t ev : ctx->free_events) cudaEventDestroy(ev);
+    if (ctx->done != nullptr) cudaEventDestroy(ctx->done);
+    if (ctx->d_partials != nullptr) cudaFree(ctx->d_partials);
+    if (ctx->d_out != nullptr) cudaFree(ctx->d_out);
+    if (ctx->h_out != nullptr) cudaFreeHost(ctx->h_out);
+    delete ctx;
+}
+
+int adpsgd_local_steps(adpsgd_ctx* ctx, int64_t k0, int32_t m, const float* lr)
+{
+    if (ctx == nullptr || m < 0 || k0 < 0 || k0 + m > kMaxK || (m > 0 && lr == nullptr)) return ADPSGD_E_INVAL;
+    for (int32_t t = 0; t < m; ++t) {
+        int st = local_step(ctx, k0 + t, lr[t]);
+        if (st != ADPSGD_OK) return st;
+    }
+    return ADPSGD_OK;
+}
+
+int adpsgd_average_and_variance(adpsgd_ctx* ctx, double* D_out, double* loss_out)
+{
+    if (ctx == nullptr || D_out == nullptr) return ADPSGD_E_INVAL;
+    if (loss_out != nullptr && !ctx->cfg.want_loss) return ADPSGD_E_STATE;
+    int st = average(ctx, true, loss_out != nullptr);
+    if (st != ADPSGD_OK) return st;
+    *D_out = ctx->h_out[0];
+    if (loss_out != nullptr) *loss_out = ctx->h_out[1];
+    return ADPSGD_OK;
+}
+
+int adpsgd_variance(adpsgd_ctx* ctx, double* D_out)
+{
+    if (ctx == nullptr || D_out == nullptr) return ADPSGD_E_INVAL;
+    int st = average(ctx, false, false);
+    if (st != ADPSGD_OK) return st;
+    *D_out = ctx->h_out[0];
+    return ADPSGD_OK;
+}
+
+int adpsgd_state_init(const adpsgd_schedule* sched, adpsgd_state* state)
+{
+    if (state == nullptr || check_schedule(sched) != ADPSGD_OK) return ADPSGD_E_INVAL;
+    state->k_next = 0;
+    state->cnt = 0;
+    state->p = sched->p_init;
+    state->C2 = 0.0;
+    state->m = 0;
+    state->rounds = 0;
+    return ADPSGD_OK;
+}
+
+int adpsgd_sched_on_sync(const adpsgd_schedule* sched, adpsgd_state* state, int64_t k, double S,
+                         double gamma, int32_t* phase)
+{
+    if (state == nullptr || check_schedule(sched) != ADPSGD_OK || !(gamma > 0.0)) return ADPSGD_E_INVAL;
+    int32_t ph = rule(sched, state, k, S, gamma);
+    if (phase != nullptr) *phase = ph;
+    return ADPSGD_OK;
+}
+
+int adpsgd_gamma(const adpsgd_schedule* sched, int64_t k, float* gamma_out)
+{
+    if (gamma_out == nullptr || check_schedule(sched) != ADPSGD_OK || k < 0) return ADPSGD_E_INVAL;
+    *gamma_out = gamma_of(sched, k);
+    return ADPSGD_OK;
+}
+
+int adpsgd_wire_bytes(int32_t n, int64_t P, int64_t rounds, int32_t with_scalar, double* per_node,
+                      double* total)
+{
+    if (n < 1 || P < 0 || rounds < 0 || per_node == nullptr || total == nullptr) return ADPSGD_E_INVAL;
+    wire(n, P, rounds, with_scalar != 0, per_node, total);
+    return ADPSGD_OK;
+}
+
+int adpsgd_run(adpsgd_ctx* ctx, const adpsgd_schedule* sched, adpsgd_state* state, int64_t k_end,
+               adpsgd_trace* trace, adpsgd_stats* stats)
+{
+    if (ctx == nullptr || state == nullptr) return ADPSGD_E_INVAL;
+    int st = check_schedule(sched);
+    if (st != ADPSGD_OK) return st;
+    if (state->p < 1 || state->k_next < 0 || state->cnt < 0) return ADPSGD_E_INVAL;
+    if (trace != nullptr && (trace->cap < 0 || (trace->cap > 0 && (trace->k == nullptr || trace->p == nullptr ||
+                                                                    trace->S == nullptr || trace->C2 == nullptr ||
+                                                                    trace->loss == nullptr || trace->phase == nullptr))))
+        return ADPSGD_E_INVAL;
+    const bool loss = ctx->cfg.want_loss != 0;
+    const int64_t stop = k_end < sched->K ? k_end : sched->K;
+    const int64_t launches0[2] = {ctx->launches[0], ctx->launches[1]};
+    for (int64_t k = state->k_next; k < stop; ++k) {
+        const float gamma = gamma_of(sched, k);
+        st = local_step(ctx, k, gamma);
+        if (st != ADPSGD_OK) return st;
+        state->k_next = k + 1;
+        if (!sync_after(sched, state, k)) continue;
+        st = average(ctx, true, loss);
+        if (st != ADPSGD_OK) return st;
+        const double S = ctx->h_out[0] / (double)ctx->cfg.n;
+        const int32_t phase = rule(sched, state, k, S, (double)gamma);
+        if (trace != nullptr) {
+            if (trace->len < trace->cap) {
+                const int64_t t = trace->len;
+                trace->k[t] = k;
+                trace->p[t] = state->p;
+                trace->S[t] = S;
+                trace->C2[t] = state->C2;
+                trace->loss[t] = loss ? ctx->h_out[1] : 0.0;
+                trace->phase[t] = phase;
+                trace->len = t + 1;
+            }
+        }
+        state->rounds += 1;
+    }
+    if (stats != nullptr) {
+        stats->rounds = state->rounds;
+        stats->equiv_period = state->rounds > 0 ? (double)state->k_next / (double)state->rounds : 0.0;
+        double total = 0.0;
+        wire(ctx->cfg.n, ctx->cfg.P, state->rounds, true, &stats->wire_bytes_per_node, &stats->wire_bytes_total);
+        wire(ctx->cfg.n, ctx->cfg.P, state->k_next, false, &stats->fullsgd_wire_bytes_per_node, &total);
+        stats->local_step_launches = ctx->launches[0] - launches0[0];
+        stats->average_launches = ctx->launches[1] - launches0[1];
+    }
+    return ADPSGD_OK;
+}
+
+int adpsgd_philox_fill(uint64_t seed, uint32_t tag, int32_t n, int64_t nq, int64_t k, uint32_t* out, void* stream)
+{
+    if (out == nullptr || n < 0 || nq < 0 || nq > kMaxK || k < 0 || k >= kMaxK) return ADPSGD_E_INVAL;
+    if (!aligned16(out)) return ADPSGD_E_ALIGN;
+    cudaError_t e = adpsgd::launch_philox_fill(seed, tag, n, nq, (uint32_t)k, out, static_cast<cudaStream_t>(stream));
+    return e == cudaSuccess ? ADPSGD_OK : cuda_fail(e, "philox fill");
+}
+
+int adpsgd_noise_fill_f32(uint64_t seed, uint32_t tag, int32_t n, int64_t P, int64_t k, float* out, void* stream)
+{
+    if (out == nullptr || n < 0 || P < 0 || P > (int64_t(1) << 34) || k < 0 || k >= kMaxK) return ADPSGD_E_INVAL;
+    if (!aligned16(out)) return ADPSGD_E_ALIGN;
+    cudaError_t e = adpsgd::launch_noise_f32(seed, tag, n, P, (uint32_t)k, out, static_cast<cudaStream_t>(stream));
+    return e == cudaSuccess ? ADPSGD_OK : cuda_fail(e, "noise fill");
+}
+
+int adpsgd_noise_fill_bf16(uint64_t seed, int32_t n, int64_t P, uint16_t* out, void* stream)
+{
+    if (out == nullptr || n < 0 || P < 0 || P > (int64_t(1) << 34)) return ADPSGD_E_INVAL;
+    if (!aligned16(out)) return ADPSGD_E_ALIGN;
+    cudaError_t e = adpsgd::launch_noise_bf16(seed, n, P, out, static_cast<cudaStream_t>(stream));
+    return e == cudaSuccess ? ADPSGD_OK : cuda_fail(e, "bf16 noise fill");
+}
+
+int adpsgd_kernel_times(adpsgd_ctx* ctx, double* local_step_ms, int64_t* local_step_launches, double* average_ms,
+                        int64_t* average_launches)
+{
+    if (ctx == nullptr) return ADPSGD_E_INVAL;
+    if (!ctx->cfg.time_kernels) return ADPSGD_E_STATE;
+    int st = harvest_times(ctx);
+    if (st != ADPSGD_OK) return st;
+    if (local_step_ms != nullptr) *local_step_ms = ctx->ms[0];
+    if (local_step_launches != nullptr) *local_step_launches = ctx->timed_launches[0];
+    if (average_ms != nullptr) *average_ms = ctx->ms[1];
+    if (average_launches != nullptr) *average_launches = ctx->timed_launches[1];
+    return ADPSGD_OK;
+}
+
+int adpsgd_reset_kernel_times(adpsgd_ctx* ctx)
+{
+    if (ctx == nullptr) return ADPSGD_E_INVAL;
+    if (ctx->cfg.time_kernels) {
+        int st = harvest_times(ctx);
+        if (st != ADPSGD_OK) return st;
+    }
+    ctx->ms[0] = ctx->ms[1] = 0.0;
+    ctx->timed_launches[0] = ctx->timed_launches[1] = 0;
+    return ADPSGD_OK;
+}
+
+int adpsgd_test_force_incomplete(adpsgd_ctx* ctx, int32_t force_incomplete)
+{
+    if (ctx == nullptr) return ADPSGD_E_INVAL;
+    ctx->force_incomplete = force_incomplete != 0;
+    return ADPSGD_OK;
+}
+
+}  // extern "C"
