@@ -39,7 +39,7 @@ sys.path.insert(0, ROOT)
 METRIC = "avg+variance GB/s vs HBM peak; fused local-step replica-params/sec"
 UNIT = "replica-params/s"
 CPU_SAMPLE_COLUMNS = 1 << 20
-CPU_SAMPLE_ITERS = 8
+CPU_SAMPLE_ITERS = 24
 
 
 def log(*a):
@@ -55,18 +55,34 @@ def measured_peaks():
     return 6800.0, "fallback"
 
 
+KERNEL_SOURCES = {
+    # kernel -> (file, first line marker, end marker) of the source it is built from
+    "local_step_kernel": [("kernels.cu", "struct StepParams", "struct AvgParams"), ("noise.cuh", "", "")],
+    "average_kernel": [("kernels.cu", "struct AvgParams", "__global__ void __launch_bounds__(kThreads) philox_fill")],
+}
+
+
+def kernel_source_digest(kernel: str) -> str:
+    """sha256 (16 hex) of the source text a kernel is compiled from."""
+    import hashlib
+    h = hashlib.sha256()
+    for fname, begin, end in KERNEL_SOURCES[kernel]:
+        text = open(os.path.join(ROOT, "paper_2007_06134_gb300", "csrc", fname)).read()
+        a = text.index(begin) if begin else 0
+        b = text.index(end, a) if end else len(text)
+        h.update(text[a:b].encode())
+    return h.hexdigest()[:16]
+
+
 def recorded_traffic(kernel: str, workload: str):
     """DRAM bytes per launch from a committed ncu capture, if the kernel source is unchanged since."""
     path = os.path.join(ROOT, "profiles", "traffic.json")
     if not os.path.exists(path):
         return None
-    import hashlib
     with open(path) as f:
         d = json.load(f)
-    src = os.path.join(ROOT, "paper_2007_06134_gb300", "csrc", "kernels.cu")
-    digest = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
     e = d.get(kernel, {}).get(workload)
-    if not e or e.get("kernels_cu_sha256_16") != digest:
+    if not e or e.get("source_sha256_16") != kernel_source_digest(kernel):
         return None
     return e["dram_bytes_per_launch"]
 
@@ -412,13 +428,19 @@ def main():
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=["gb300", "reference"], default="gb300")
     ap.add_argument("--workload", default="resnet18-n8")
+    ap.add_argument("--iters", type=int, default=None,
+                    help="override the workload's iteration count (profiling captures only)")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu", action="store_true")
     ap.add_argument("--sweep", action="store_true", help="averaging-kernel sweep over n x P instead")
-    ap.add_argument("--sweep-max-bytes", type=float, default=34e9)
+    ap.add_argument("--sweep-max-bytes", type=float, default=70e9)
     args = ap.parse_args()
     from paper_2007_06134_gb300 import inputs
     w = inputs.WORKLOADS[args.workload]
+    if args.iters is not None:
+        import dataclasses
+        w = dataclasses.replace(w, K=args.iters, K_s_frac=min(w.K_s_frac, 0.5),
+                                milestones=tuple(int(m * args.iters / w.K) for m in w.milestones))
     if args.impl == "reference":
         return run_reference(args, w)
     if args.sweep:
