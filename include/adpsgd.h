@@ -145,6 +145,31 @@ int adpsgd_local_steps(adpsgd_ctx* ctx, int64_t k0, int32_t m, const float* lr);
  * Errors: E_INVAL (D_out NULL), E_STATE (loss requested without want_loss), E_TIMEOUT, E_CUDA. */
 int adpsgd_average_and_variance(adpsgd_ctx* ctx, double* D_out, double* loss_out);
 
+/* The same averaging as adpsgd_average_and_variance, for callers that cannot allocate device
+ * memory: code running inside a host framework whose pool allocator owns the GPU's memory
+ * (a cudaMalloc of its own would bypass or fragment that pool), and code on a latency-critical
+ * path where cudaMalloc / cudaFree would synchronise the device.  The paper has no counterpart:
+ * this is an interface variant, not part of the method.
+ *
+ * It needs no context and allocates nothing.  Its scratch is a fixed array inside the library,
+ * 2 * 2048 + 2 doubles (32.8 KB), which every GPU that loads the library holds until the process
+ * exits.  The per-block partial sums for up to 2048 blocks live there.  A shape whose averaging
+ * grid would need more blocks is rejected with ADPSGD_E_INVAL; on GB300 the grid is at most
+ * 1216 blocks.
+ *
+ * x: device fp32 [n, P], read, then xbar written to every row.  h, c: device fp32 [P], needed
+ * only when loss_out != NULL.  D_out, loss_out: host doubles; loss_out may be NULL.
+ * stream: cudaStream_t as void*.  wait_timeout_ms bounds the wait for the stream (<= 0: 60000).
+ *
+ * The first call on each device looks up the scratch array's device address
+ * (cudaGetSymbolAddress).  Make that first call before any stream capture.  Every call uses the
+ * same array, which keeps the last call's contents.  Each call writes every slot it later reads,
+ * so nothing needs clearing between calls.  Calls that overlap on the GPU (several host threads,
+ * or streams that run concurrently) race on the array and must be serialised by the caller.
+ * Errors: E_INVAL, E_ALIGN, E_TIMEOUT, E_CUDA. */
+int adpsgd_average_and_variance_static(float* x, const float* h, const float* c, int32_t n, int64_t P,
+                                       double* D_out, double* loss_out, int64_t wait_timeout_ms, void* stream);
+
 /* D = sum_j sum_i (x_ij - xbar_j)^2 without averaging (the per-iteration Var[W_k] of
  * Sec. III and Eq. vt, times n).  Blocks (bounded).  Errors: as above. */
 int adpsgd_variance(adpsgd_ctx* ctx, double* D_out);

@@ -68,6 +68,8 @@ _SIGS = {
     "adpsgd_local_steps": (C.c_int, [_P, C.c_int64, C.c_int32, C.POINTER(C.c_float)]),
     "adpsgd_average_and_variance": (C.c_int, [_P, C.POINTER(C.c_double), C.POINTER(C.c_double)]),
     "adpsgd_variance": (C.c_int, [_P, C.POINTER(C.c_double)]),
+    "adpsgd_average_and_variance_static": (C.c_int, [_P, _P, _P, C.c_int32, C.c_int64, C.POINTER(C.c_double),
+                                                     C.POINTER(C.c_double), C.c_int64, _P]),
     "adpsgd_state_init": (C.c_int, [C.POINTER(Schedule), C.POINTER(State)]),
     "adpsgd_run": (C.c_int, [_P, C.POINTER(Schedule), C.POINTER(State), C.c_int64, C.POINTER(Trace),
                              C.POINTER(Stats)]),
@@ -206,6 +208,18 @@ def adpsgd_average_and_variance(ctx: Context, want_loss: bool = True):
     L = C.c_double()
     _check(load().adpsgd_average_and_variance(ctx.handle, C.byref(D), C.byref(L) if want_loss else None),
            "adpsgd_average_and_variance")
+    return D.value, (L.value if want_loss else None)
+
+
+def adpsgd_average_and_variance_static(x, h, c, n: int, P: int, want_loss: bool = True,
+                                       wait_timeout_ms: int = 60000, stream=None):
+    """Averaging without a context or any allocation (fixed scratch inside the library)."""
+    D = C.c_double()
+    L = C.c_double()
+    _check(load().adpsgd_average_and_variance_static(_ptr(x), _ptr(h), _ptr(c), n, P, C.byref(D),
+                                                     C.byref(L) if want_loss else None, wait_timeout_ms,
+                                                     _stream(stream)),
+           "adpsgd_average_and_variance_static")
     return D.value, (L.value if want_loss else None)
 
 

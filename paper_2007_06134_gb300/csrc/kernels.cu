@@ -20,6 +20,8 @@
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 
+#include <mutex>
+
 #include "launch.h"
 #include "noise.cuh"
 
@@ -473,6 +475,48 @@ cudaError_t launch_noise_bf16(uint64_t seed, int32_t n, int64_t P, uint16_t* out
     if (blocks == 0) return cudaSuccess;
     noise_bf16_kernel<<<(unsigned)blocks, kThreads, 0, stream>>>(keys, n, P, Q, out);
     return cudaGetLastError();
+}
+
+// ------------------------------------------------------------------------------------------
+// Fixed device scratch for the averaging entry point that allocates nothing
+// ------------------------------------------------------------------------------------------
+// The partial sums of up to kStaticMaxBlocks blocks (D then loss) followed by the two finished
+// sums: 2 * 2048 + 2 doubles = 32.8 KB, held by every GPU that loads this library until exit.
+constexpr int kStaticMaxBlocks = 2048;
+constexpr int kStaticMaxDevices = 64;
+
+}  // namespace adpsgd
+
+static __device__ __align__(256) double g_static_scratch[2 * adpsgd::kStaticMaxBlocks + 2];
+
+namespace adpsgd {
+
+namespace {
+std::mutex g_static_mutex;
+double* g_static_address[kStaticMaxDevices] = {};
+}  // namespace
+
+int static_scratch_max_blocks() { return kStaticMaxBlocks; }
+
+// Device address of g_static_scratch on the current device.  On host, the symbol's name is
+// only a stand-in, not a device address, so it is looked up once per device (with that device
+// current) and cached.
+cudaError_t static_scratch_address(double** partials, double** out)
+{
+    int device = 0;
+    cudaError_t e = cudaGetDevice(&device);
+    if (e != cudaSuccess) return e;
+    if (device < 0 || device >= kStaticMaxDevices) return cudaErrorInvalidDevice;
+    std::lock_guard<std::mutex> lock(g_static_mutex);
+    if (g_static_address[device] == nullptr) {
+        void* address = nullptr;
+        e = cudaGetSymbolAddress(&address, g_static_scratch);
+        if (e != cudaSuccess) return e;
+        g_static_address[device] = static_cast<double*>(address);
+    }
+    *partials = g_static_address[device];
+    *out = g_static_address[device] + 2 * kStaticMaxBlocks;
+    return cudaSuccess;
 }
 
 }  // namespace adpsgd

@@ -50,6 +50,11 @@ cudaError_t launch_average(const AverageArgs& a, cudaStream_t stream);
 int average_grid(int32_t n, int64_t P, bool loss, bool write_back, int sms);
 int average_grid_max(int sms);
 
+// Fixed device scratch (no allocation): partial sums for up to static_scratch_max_blocks()
+// blocks and the two finished sums.  The first call on a device looks the address up.
+int static_scratch_max_blocks();
+cudaError_t static_scratch_address(double** partials, double** out);
+
 cudaError_t launch_philox_fill(uint64_t seed, uint32_t tag, int32_t n, int64_t nq, uint32_t k,
                                uint32_t* out, cudaStream_t stream);
 cudaError_t launch_noise_f32(uint64_t seed, uint32_t tag, int32_t n, int64_t P, uint32_t k,

@@ -459,6 +459,60 @@ int adpsgd_run(adpsgd_ctx* ctx, const adpsgd_schedule* sched, adpsgd_state* stat
     return ADPSGD_OK;
 }
 
+int adpsgd_average_and_variance_static(float* x, const float* h, const float* c, int32_t n, int64_t P,
+                                       double* D_out, double* loss_out, int64_t wait_timeout_ms, void* stream)
+{
+    if (x == nullptr || D_out == nullptr || n < 1 || P < 1) return ADPSGD_E_INVAL;
+    if (P > (int64_t(1) << 34) || (int64_t)n * P > (int64_t(1) << 40)) return ADPSGD_E_INVAL;
+    const bool loss = loss_out != nullptr;
+    if (loss && (h == nullptr || c == nullptr)) return ADPSGD_E_INVAL;
+    if (!aligned16(x) || (loss && (!aligned16(h) || !aligned16(c)))) return ADPSGD_E_ALIGN;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    int device = 0, sms = 0;
+    cudaError_t e = cudaGetDevice(&device);
+    if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, device);
+    if (e != cudaSuccess) return cuda_fail(e, "device query");
+    const int grid = adpsgd::average_grid(n, P, loss, true, sms);
+    if (grid > adpsgd::static_scratch_max_blocks()) {
+        g_last_error = "the averaging grid needs " + std::to_string(grid) + " partial-sum slots; the fixed scratch holds " +
+                       std::to_string(adpsgd::static_scratch_max_blocks());
+        return ADPSGD_E_INVAL;
+    }
+    adpsgd::AverageArgs a;
+    a.x = x;
+    a.h = loss ? h : nullptr;
+    a.c = loss ? c : nullptr;
+    a.n = n;
+    a.P = P;
+    a.write_back = true;
+    a.grid = grid;
+    e = adpsgd::static_scratch_address(&a.partials, &a.out);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaGetSymbolAddress");
+    e = adpsgd::launch_average(a, s);
+    if (e != cudaSuccess) return cuda_fail(e, "average");
+    // Bounded wait for the stream, then a 16-byte copy from an idle stream.
+    const auto t0 = std::chrono::steady_clock::now();
+    const auto limit = std::chrono::milliseconds(wait_timeout_ms > 0 ? wait_timeout_ms : 60000);
+    int spins = 0;
+    for (;;) {
+        e = cudaStreamQuery(s);
+        if (e == cudaSuccess) break;
+        if (e != cudaErrorNotReady) return cuda_fail(e, "cudaStreamQuery");
+        if (std::chrono::steady_clock::now() - t0 > limit) {
+            g_last_error = "bounded wait ran out";
+            return ADPSGD_E_TIMEOUT;
+        }
+        if (++spins > 2000) std::this_thread::sleep_for(std::chrono::microseconds(20));
+    }
+    double result[2] = {0.0, 0.0};
+    e = cudaMemcpyAsync(result, a.out, sizeof(result), cudaMemcpyDeviceToHost, s);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaMemcpyAsync");
+    *D_out = result[0];
+    if (loss) *loss_out = result[1];
+    return ADPSGD_OK;
+}
+
 int adpsgd_philox_fill(uint64_t seed, uint32_t tag, int32_t n, int64_t nq, int64_t k, uint32_t* out, void* stream)
 {
     if (out == nullptr || n < 0 || nq < 0 || nq > kMaxK || k < 0 || k >= kMaxK) return ADPSGD_E_INVAL;
