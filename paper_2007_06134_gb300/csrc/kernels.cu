@@ -9,9 +9,9 @@
 //   average_kernel     Algorithm 2 averaging + S_k: per column, the replica mean, the squared
 //                      deviations and the surrogate loss, x̄ written back to every replica;
 //                      replica values of a column stay in registers between the passes.
-//                      Persistent grid; each block leaves one fp64 partial per sum, and a
-//                      one-block kernel adds the partials in a fixed order (deterministic,
-//                      no inter-block wait).  HBM-bound: 8 B per replica-param.
+//                      Persistent grid; each block leaves one fp64 partial per sum and the
+//                      last block to finish adds them in block order (deterministic; an
+//                      atomic ticket, no inter-block wait).  HBM-bound: 8 B per replica-param.
 //   *_fill kernels     the raw Philox stream, its fp32 normals, and the bf16 noise tensor.
 //
 // Every fp32 operation of the update, the mean and the generator is written out once and
@@ -141,9 +141,11 @@ struct AvgParams {
     const float* h;
     const float* c;
     int64_t P;
-    int64_t Q;  // columns (scalar) or blocks of four columns (vector) handled by one thread
+    int64_t Q;  // column groups: blocks of four columns (vector) or single columns (scalar)
     int32_t n;
-    double* partials;
+    double* partials;       // 2 * gridDim.x: per-block D, then per-block loss
+    double* out;            // out[0] = D, out[1] = loss
+    unsigned int* counter;  // zero at launch; the last block to finish sets it back to zero
 };
 
 // Fixed-order block sum; the result is valid in thread 0.
@@ -198,73 +200,117 @@ __device__ __forceinline__ void column_stats_global(const float* x, int64_t P, i
     d = s;
 }
 
-template <int NMAX, bool VEC, bool LOSS, bool WRITE>
-__global__ void __launch_bounds__(kThreads) average_kernel(const AvgParams p)
+// A column group is one float4 (four columns) of every replica, or one float (scalar rows).
+template <bool VEC> struct ColumnGroup;
+template <> struct ColumnGroup<true> {
+    using T = float4;
+    static constexpr int W = 4;
+    static __device__ __forceinline__ float lane(const float4& v, int r)
+    {
+        return r == 0 ? v.x : (r == 1 ? v.y : (r == 2 ? v.z : v.w));
+    }
+    static __device__ __forceinline__ float4 make(const float* f) { return make_float4(f[0], f[1], f[2], f[3]); }
+};
+template <> struct ColumnGroup<false> {
+    using T = float;
+    static constexpr int W = 1;
+    static __device__ __forceinline__ float lane(float v, int) { return v; }
+    static __device__ __forceinline__ float make(const float* f) { return f[0]; }
+};
+
+// Statistics, loss and write-back of column group q whose replica values are vals[0..n).
+template <int R, bool VEC, bool LOSS, bool WRITE>
+__device__ __forceinline__ void finish_group(const AvgParams& p, int64_t q, const typename ColumnGroup<VEC>::T* vals,
+                                             float nf, double& accD, double& accL)
 {
+    using G = ColumnGroup<VEC>;
+    constexpr int W = G::W;
+    float xbar[W], d[W];
+#pragma unroll
+    for (int r = 0; r < W; ++r) {
+        float col[R];
+#pragma unroll
+        for (int i = 0; i < R; ++i) col[i] = (i < p.n) ? G::lane(vals[i], r) : 0.0f;
+        column_stats<R>(col, p.n, nf, xbar[r], d[r]);
+    }
+    accD += VEC ? (double)((d[0] + d[W > 1 ? 1 : 0]) + (d[W > 2 ? 2 : 0] + d[W > 3 ? 3 : 0])) : (double)d[0];
+    if (LOSS) {
+        const typename G::T hv = reinterpret_cast<const typename G::T*>(p.h)[q];
+        const typename G::T cv = reinterpret_cast<const typename G::T*>(p.c)[q];
+        float l[W];
+#pragma unroll
+        for (int r = 0; r < W; ++r) {
+            const float t = xbar[r] - G::lane(cv, r);
+            l[r] = (G::lane(hv, r) * t) * t;
+        }
+        accL += VEC ? (double)((l[0] + l[W > 1 ? 1 : 0]) + (l[W > 2 ? 2 : 0] + l[W > 3 ? 3 : 0])) : (double)l[0];
+    }
+    if (WRITE) {
+        const typename G::T out = G::make(xbar);
+#pragma unroll
+        for (int i = 0; i < R; ++i)
+            if (i < p.n) reinterpret_cast<typename G::T*>(p.x + (int64_t)i * p.P)[q] = out;
+    }
+}
+
+// Persistent grid over column groups; each thread keeps the n replica values of U groups in
+// registers (NMAX >= n), so the loads of U groups are in flight together.  NMAX = 0: any n,
+// values re-read per pass.  The block partials are added by the last block to finish, in
+// block order, so the sums do not depend on which block finishes last.
+template <int NMAX, int U, bool VEC, bool LOSS, bool WRITE>
+__global__ void __launch_bounds__(kThreads, (NMAX >= 32 ? 1 : 2)) average_kernel(const AvgParams p)
+{
+    using G = ColumnGroup<VEC>;
+    using T = typename G::T;
     __shared__ double shared[kThreads / 32];
-    const int32_t n = p.n;
-    const float nf = (float)n;
+    __shared__ unsigned int ticket;
+    const float nf = (float)p.n;
     double accD = 0.0, accL = 0.0;
     const int64_t stride = (int64_t)gridDim.x * kThreads;
-    for (int64_t q = (int64_t)blockIdx.x * kThreads + threadIdx.x; q < p.Q; q += stride) {
-        if (VEC) {
-            float xbar[4], d[4];
-            if (NMAX > 0) {
-                constexpr int R = NMAX > 0 ? NMAX : 1;
-                float4 r4[R];
+    for (int64_t q0 = (int64_t)blockIdx.x * kThreads + threadIdx.x; q0 < p.Q; q0 += U * stride) {
+        if (NMAX > 0) {
+            constexpr int R = NMAX > 0 ? NMAX : 1;
+            T vals[U][R];
 #pragma unroll
-                for (int i = 0; i < R; ++i)
-                    if (i < n) r4[i] = reinterpret_cast<const float4*>(p.x + (int64_t)i * p.P)[q];
-                float col[R];
+            for (int u = 0; u < U; ++u) {
+                const int64_t q = q0 + u * stride;
+                if (q < p.Q) {
 #pragma unroll
-                for (int i = 0; i < R; ++i) col[i] = (i < n) ? r4[i].x : 0.0f;
-                column_stats<R>(col, n, nf, xbar[0], d[0]);
-#pragma unroll
-                for (int i = 0; i < R; ++i) col[i] = (i < n) ? r4[i].y : 0.0f;
-                column_stats<R>(col, n, nf, xbar[1], d[1]);
-#pragma unroll
-                for (int i = 0; i < R; ++i) col[i] = (i < n) ? r4[i].z : 0.0f;
-                column_stats<R>(col, n, nf, xbar[2], d[2]);
-#pragma unroll
-                for (int i = 0; i < R; ++i) col[i] = (i < n) ? r4[i].w : 0.0f;
-                column_stats<R>(col, n, nf, xbar[3], d[3]);
-            } else {
-#pragma unroll
-                for (int r = 0; r < 4; ++r) column_stats_global(p.x, p.P, 4 * q + r, n, nf, xbar[r], d[r]);
+                    for (int i = 0; i < R; ++i)
+                        if (i < p.n) vals[u][i] = reinterpret_cast<const T*>(p.x + (int64_t)i * p.P)[q];
+                }
             }
-            accD += (double)((d[0] + d[1]) + (d[2] + d[3]));
-            if (LOSS) {
-                const float4 hv = __ldg(reinterpret_cast<const float4*>(p.h) + q);
-                const float4 cv = __ldg(reinterpret_cast<const float4*>(p.c) + q);
-                const float t0 = xbar[0] - cv.x, t1 = xbar[1] - cv.y, t2 = xbar[2] - cv.z, t3 = xbar[3] - cv.w;
-                const float l0 = (hv.x * t0) * t0, l1 = (hv.y * t1) * t1;
-                const float l2 = (hv.z * t2) * t2, l3 = (hv.w * t3) * t3;
-                accL += (double)((l0 + l1) + (l2 + l3));
-            }
-            if (WRITE) {
-                const float4 out = make_float4(xbar[0], xbar[1], xbar[2], xbar[3]);
-                for (int i = 0; i < n; ++i) reinterpret_cast<float4*>(p.x + (int64_t)i * p.P)[q] = out;
+#pragma unroll
+            for (int u = 0; u < U; ++u) {
+                const int64_t q = q0 + u * stride;
+                if (q < p.Q) finish_group<R, VEC, LOSS, WRITE>(p, q, vals[u], nf, accD, accL);
             }
         } else {
-            const int64_t j = q;
-            float xbar, d;
-            if (NMAX > 0) {
-                constexpr int R = NMAX > 0 ? NMAX : 1;
-                float col[R];
+            const int64_t q = q0;
+            float xbar[G::W], d[G::W];
 #pragma unroll
-                for (int i = 0; i < R; ++i) col[i] = (i < n) ? p.x[(int64_t)i * p.P + j] : 0.0f;
-                column_stats<R>(col, n, nf, xbar, d);
-            } else {
-                column_stats_global(p.x, p.P, j, n, nf, xbar, d);
-            }
-            accD += (double)d;
+            for (int r = 0; r < G::W; ++r) column_stats_global(p.x, p.P, G::W * q + r, p.n, nf, xbar[r], d[r]);
+            double dsum = 0.0;
+            float fsum = 0.0f;
+            if (VEC) fsum = (d[0] + d[G::W > 1 ? 1 : 0]) + (d[G::W > 2 ? 2 : 0] + d[G::W > 3 ? 3 : 0]);
+            dsum = VEC ? (double)fsum : (double)d[0];
+            accD += dsum;
             if (LOSS) {
-                const float t = xbar - __ldg(p.c + j);
-                const float l = (__ldg(p.h + j) * t) * t;
-                accL += (double)l;
+                const T hv = reinterpret_cast<const T*>(p.h)[q];
+                const T cv = reinterpret_cast<const T*>(p.c)[q];
+                float l[G::W];
+#pragma unroll
+                for (int r = 0; r < G::W; ++r) {
+                    const float t = xbar[r] - G::lane(cv, r);
+                    l[r] = (G::lane(hv, r) * t) * t;
+                }
+                accL += VEC ? (double)((l[0] + l[G::W > 1 ? 1 : 0]) + (l[G::W > 2 ? 2 : 0] + l[G::W > 3 ? 3 : 0]))
+                            : (double)l[0];
             }
-            if (WRITE)
-                for (int i = 0; i < n; ++i) p.x[(int64_t)i * p.P + j] = xbar;
+            if (WRITE) {
+                const T out = G::make(xbar);
+                for (int i = 0; i < p.n; ++i) reinterpret_cast<T*>(p.x + (int64_t)i * p.P)[q] = out;
+            }
         }
     }
     const double bD = block_sum(accD, shared);
@@ -272,23 +318,24 @@ __global__ void __launch_bounds__(kThreads) average_kernel(const AvgParams p)
     if (threadIdx.x == 0) {
         p.partials[blockIdx.x] = bD;
         p.partials[gridDim.x + blockIdx.x] = bL;
+        __threadfence();
+        ticket = atomicAdd(p.counter, 1u);
     }
-}
-
-// out[0] = sum of the D partials, out[1] = 1/2 sum of the loss partials, in a fixed order.
-__global__ void __launch_bounds__(kThreads) finalize_kernel(const double* partials, int nblocks, double* out)
-{
-    __shared__ double shared[kThreads / 32];
+    __syncthreads();
+    if (ticket != gridDim.x - 1) return;
+    // The last block: every other block's partials are visible (fence before each increment).
+    __threadfence();
     double d = 0.0, l = 0.0;
-    for (int b = threadIdx.x; b < nblocks; b += kThreads) {
-        d += partials[b];
-        l += partials[nblocks + b];
+    for (int b = threadIdx.x; b < (int)gridDim.x; b += kThreads) {
+        d += __ldcg(p.partials + b);
+        if (LOSS) l += __ldcg(p.partials + gridDim.x + b);
     }
     d = block_sum(d, shared);
-    l = block_sum(l, shared);
+    if (LOSS) l = block_sum(l, shared);
     if (threadIdx.x == 0) {
-        out[0] = d;
-        out[1] = 0.5 * l;
+        p.out[0] = d;
+        p.out[1] = 0.5 * l;
+        *p.counter = 0u;
     }
 }
 
@@ -344,24 +391,26 @@ int max_blocks_per_sm(Kernel kernel)
 
 using AvgKernel = void (*)(const AvgParams);
 
-template <int NMAX>
+template <int NMAX, int U>
 AvgKernel pick_average_nmax(bool vec, bool loss, bool write)
 {
     if (vec) {
-        if (!write) return average_kernel<NMAX, true, false, false>;
-        return loss ? average_kernel<NMAX, true, true, true> : average_kernel<NMAX, true, false, true>;
+        if (!write) return average_kernel<NMAX, U, true, false, false>;
+        return loss ? average_kernel<NMAX, U, true, true, true> : average_kernel<NMAX, U, true, false, true>;
     }
-    if (!write) return average_kernel<NMAX, false, false, false>;
-    return loss ? average_kernel<NMAX, false, true, true> : average_kernel<NMAX, false, false, true>;
+    if (!write) return average_kernel<NMAX, U, false, false, false>;
+    return loss ? average_kernel<NMAX, U, false, true, true> : average_kernel<NMAX, U, false, false, true>;
 }
 
+// Register-resident variants: NMAX replicas x U column groups per thread (NMAX * U <= 32 float4).
 AvgKernel pick_average(int32_t n, bool vec, bool loss, bool write)
 {
-    if (n <= 4) return pick_average_nmax<4>(vec, loss, write);
-    if (n <= 8) return pick_average_nmax<8>(vec, loss, write);
-    if (n <= 16) return pick_average_nmax<16>(vec, loss, write);
-    if (n <= 32) return pick_average_nmax<32>(vec, loss, write);
-    return pick_average_nmax<0>(vec, loss, write);
+    if (n <= 2) return pick_average_nmax<2, 8>(vec, loss, write);
+    if (n <= 4) return pick_average_nmax<4, 4>(vec, loss, write);
+    if (n <= 8) return pick_average_nmax<8, 2>(vec, loss, write);
+    if (n <= 16) return pick_average_nmax<16, 1>(vec, loss, write);
+    if (n <= 32) return pick_average_nmax<32, 1>(vec, loss, write);
+    return pick_average_nmax<0, 1>(vec, loss, write);
 }
 
 bool use_vec(int64_t P, const void* a, const void* b, const void* c, const void* d)
@@ -435,11 +484,10 @@ cudaError_t launch_average(const AverageArgs& a, cudaStream_t stream)
     p.Q = vec ? a.P / 4 : a.P;
     p.n = a.n;
     p.partials = a.partials;
+    p.out = a.out;
+    p.counter = a.counter;
     const AvgKernel kernel = pick_average(a.n, vec, loss, a.write_back);
     kernel<<<a.grid, kThreads, 0, stream>>>(p);
-    cudaError_t e = cudaGetLastError();
-    if (e != cudaSuccess) return e;
-    finalize_kernel<<<1, kThreads, 0, stream>>>(a.partials, a.grid, a.out);
     return cudaGetLastError();
 }
 
@@ -480,14 +528,15 @@ cudaError_t launch_noise_bf16(uint64_t seed, int32_t n, int64_t P, uint16_t* out
 // ------------------------------------------------------------------------------------------
 // Fixed device scratch for the averaging entry point that allocates nothing
 // ------------------------------------------------------------------------------------------
-// The partial sums of up to kStaticMaxBlocks blocks (D then loss) followed by the two finished
-// sums: 2 * 2048 + 2 doubles = 32.8 KB, held by every GPU that loads this library until exit.
+// The partial sums of up to kStaticMaxBlocks blocks (D then loss), the two finished sums and one
+// slot for the completion counter: 2 * 2048 + 4 doubles = 32.8 KB, held by every GPU that loads
+// this library until exit.
 constexpr int kStaticMaxBlocks = 2048;
 constexpr int kStaticMaxDevices = 64;
 
 }  // namespace adpsgd
 
-static __device__ __align__(256) double g_static_scratch[2 * adpsgd::kStaticMaxBlocks + 2];
+static __device__ __align__(256) double g_static_scratch[2 * adpsgd::kStaticMaxBlocks + 4];
 
 namespace adpsgd {
 
@@ -501,7 +550,7 @@ int static_scratch_max_blocks() { return kStaticMaxBlocks; }
 // Device address of g_static_scratch on the current device.  On host, the symbol's name is
 // only a stand-in, not a device address, so it is looked up once per device (with that device
 // current) and cached.
-cudaError_t static_scratch_address(double** partials, double** out)
+cudaError_t static_scratch_address(double** partials, double** out, unsigned int** counter)
 {
     int device = 0;
     cudaError_t e = cudaGetDevice(&device);
@@ -516,6 +565,7 @@ cudaError_t static_scratch_address(double** partials, double** out)
     }
     *partials = g_static_address[device];
     *out = g_static_address[device] + 2 * kStaticMaxBlocks;
+    *counter = reinterpret_cast<unsigned int*>(g_static_address[device] + 2 * kStaticMaxBlocks + 2);
     return cudaSuccess;
 }
 

@@ -32,8 +32,9 @@ struct LocalStepArgs {
 };
 cudaError_t launch_local_step(const LocalStepArgs& a, cudaStream_t stream);
 
-// Averaging + variance (+ loss): per-block fp64 partials, then a one-block fixed-order sum
-// into out[0] (D) and out[1] (loss).
+// Averaging + variance (+ loss): per-block fp64 partials, added in block order by the last
+// block to finish into out[0] (D) and out[1] (loss).  *counter must be zero at launch; the
+// kernel leaves it zero.
 struct AverageArgs {
     float* x;
     const float* h;  // nullptr unless the loss is wanted
@@ -43,6 +44,7 @@ struct AverageArgs {
     bool write_back;  // false: variance only
     double* partials; // 2 * grid doubles
     double* out;      // 2 doubles
+    unsigned int* counter;
     int grid;         // from average_grid()
 };
 cudaError_t launch_average(const AverageArgs& a, cudaStream_t stream);
@@ -51,9 +53,9 @@ int average_grid(int32_t n, int64_t P, bool loss, bool write_back, int sms);
 int average_grid_max(int sms);
 
 // Fixed device scratch (no allocation): partial sums for up to static_scratch_max_blocks()
-// blocks and the two finished sums.  The first call on a device looks the address up.
+// blocks, the two finished sums and the completion counter.  The first call on a device looks the address up.
 int static_scratch_max_blocks();
-cudaError_t static_scratch_address(double** partials, double** out);
+cudaError_t static_scratch_address(double** partials, double** out, unsigned int** counter);
 
 cudaError_t launch_philox_fill(uint64_t seed, uint32_t tag, int32_t n, int64_t nq, uint32_t k,
                                uint32_t* out, cudaStream_t stream);

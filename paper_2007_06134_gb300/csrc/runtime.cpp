@@ -48,7 +48,7 @@ struct adpsgd_ctx {
     int sms = 0;
     adpsgd::PhiloxKeys keys{};
     double* d_partials = nullptr;
-    double* d_out = nullptr;
+    double* d_out = nullptr;  // D, loss, then the averaging kernel's completion counter
     double* h_out = nullptr;  // pinned, 2 doubles
     cudaEvent_t done = nullptr;
     int grid_avg = 0, grid_avg_loss = 0, grid_var = 0;
@@ -121,7 +121,7 @@ int timed(adpsgd_ctx* ctx, int kind, Launch launch, const char* what)
 {
     cudaEvent_t a = nullptr, b = nullptr;
     if (ctx->cfg.time_kernels) {
-        if (ctx->pending.size() >= 4096) {
+        if (ctx->pending.size() >= 16384) {
             int st = harvest_times(ctx);
             if (st != ADPSGD_OK) return st;
         }
@@ -161,8 +161,9 @@ int local_step(adpsgd_ctx* ctx, int64_t k, float gamma)
     return timed(ctx, 0, [&] { return adpsgd::launch_local_step(a, ctx->stream); }, "local step");
 }
 
-// Averaging (write_back) or variance only; results land in ctx->h_out after a bounded wait.
-int average(adpsgd_ctx* ctx, bool write_back, bool loss)
+// Enqueue the averaging (write_back) or variance-only kernel and the copy of its two sums
+// into ctx->h_out, then record ctx->done.
+int average_enqueue(adpsgd_ctx* ctx, bool write_back, bool loss)
 {
     adpsgd::AverageArgs a;
     a.x = ctx->x;
@@ -173,6 +174,7 @@ int average(adpsgd_ctx* ctx, bool write_back, bool loss)
     a.write_back = write_back;
     a.partials = ctx->d_partials;
     a.out = ctx->d_out;
+    a.counter = reinterpret_cast<unsigned int*>(ctx->d_out + 2);
     a.grid = !write_back ? ctx->grid_var : (loss ? ctx->grid_avg_loss : ctx->grid_avg);
     int st = timed(ctx, 1, [&] { return adpsgd::launch_average(a, ctx->stream); }, "average");
     if (st != ADPSGD_OK) return st;
@@ -181,10 +183,15 @@ int average(adpsgd_ctx* ctx, bool write_back, bool loss)
     if (e != cudaSuccess) return cuda_fail(e, "cudaMemcpyAsync");
     e = cudaEventRecord(ctx->done, ctx->stream);
     if (e != cudaSuccess) return cuda_fail(e, "cudaEventRecord");
-    st = wait_event(ctx, ctx->done);
-    if (st != ADPSGD_OK) return st;
-    if (ctx->cfg.time_kernels) return harvest_times(ctx);
     return ADPSGD_OK;
+}
+
+// Averaging (write_back) or variance only; results land in ctx->h_out after a bounded wait.
+int average(adpsgd_ctx* ctx, bool write_back, bool loss)
+{
+    int st = average_enqueue(ctx, write_back, loss);
+    if (st != ADPSGD_OK) return st;
+    return wait_event(ctx, ctx->done);
 }
 
 int check_schedule(const adpsgd_schedule* s)
@@ -309,7 +316,8 @@ int adpsgd_init(const adpsgd_config* cfg, float* x, float* v, const float* h, co
     ctx->grid_var = adpsgd::average_grid(cfg->n, cfg->P, false, false, ctx->sms);
     const size_t partial_bytes = 2 * sizeof(double) * (size_t)adpsgd::average_grid_max(ctx->sms);
     e = cudaMalloc(reinterpret_cast<void**>(&ctx->d_partials), partial_bytes);
-    if (e == cudaSuccess) e = cudaMalloc(reinterpret_cast<void**>(&ctx->d_out), 2 * sizeof(double));
+    if (e == cudaSuccess) e = cudaMalloc(reinterpret_cast<void**>(&ctx->d_out), 4 * sizeof(double));
+    if (e == cudaSuccess) e = cudaMemset(ctx->d_out, 0, 4 * sizeof(double));
     if (e == cudaSuccess) e = cudaMallocHost(reinterpret_cast<void**>(&ctx->h_out), 2 * sizeof(double));
     if (e == cudaSuccess) e = cudaEventCreateWithFlags(&ctx->done, cudaEventDisableTiming);
     if (e != cudaSuccess) {
@@ -423,16 +431,29 @@ int adpsgd_run(adpsgd_ctx* ctx, const adpsgd_schedule* sched, adpsgd_state* stat
     const bool loss = ctx->cfg.want_loss != 0;
     const int64_t stop = k_end < sched->K ? k_end : sched->K;
     const int64_t launches0[2] = {ctx->launches[0], ctx->launches[1]};
+    bool launched_ahead = false;  // the local step of iteration k is already enqueued
     for (int64_t k = state->k_next; k < stop; ++k) {
-        const float gamma = gamma_of(sched, k);
-        st = local_step(ctx, k, gamma);
-        if (st != ADPSGD_OK) return st;
+        if (!launched_ahead) {
+            st = local_step(ctx, k, gamma_of(sched, k));
+            if (st != ADPSGD_OK) return st;
+        }
+        launched_ahead = false;
         state->k_next = k + 1;
         if (!sync_after(sched, state, k)) continue;
-        st = average(ctx, true, loss);
+        st = average_enqueue(ctx, true, loss);
+        if (st != ADPSGD_OK) return st;
+        // Whatever the rule decides, iteration k + 1 starts with a local step (p >= 1), so it is
+        // enqueued behind the averaging before the host waits for S: the GPU stays busy while
+        // the scalars travel to the host and the rule runs.
+        if (k + 1 < stop) {
+            st = local_step(ctx, k + 1, gamma_of(sched, k + 1));
+            if (st != ADPSGD_OK) return st;
+            launched_ahead = true;
+        }
+        st = wait_event(ctx, ctx->done);
         if (st != ADPSGD_OK) return st;
         const double S = ctx->h_out[0] / (double)ctx->cfg.n;
-        const int32_t phase = rule(sched, state, k, S, (double)gamma);
+        const int32_t phase = rule(sched, state, k, S, (double)gamma_of(sched, k));
         if (trace != nullptr) {
             if (trace->len < trace->cap) {
                 const int64_t t = trace->len;
@@ -486,8 +507,11 @@ int adpsgd_average_and_variance_static(float* x, const float* h, const float* c,
     a.P = P;
     a.write_back = true;
     a.grid = grid;
-    e = adpsgd::static_scratch_address(&a.partials, &a.out);
+    e = adpsgd::static_scratch_address(&a.partials, &a.out, &a.counter);
     if (e != cudaSuccess) return cuda_fail(e, "cudaGetSymbolAddress");
+    // The array keeps the previous call's contents; the completion counter must start at zero.
+    e = cudaMemsetAsync(a.counter, 0, sizeof(unsigned int), s);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaMemsetAsync");
     e = adpsgd::launch_average(a, s);
     if (e != cudaSuccess) return cuda_fail(e, "average");
     // Bounded wait for the stream, then a 16-byte copy from an idle stream.

@@ -1,0 +1,150 @@
+"""Parity at the workloads' full sizes, in the launch configuration the bench times.
+
+The surrogate objective is separable per column and the constant-period schedule does not
+depend on the data, so the oracle can follow a full-size constant-period run exactly on a
+sample of columns: bit-exact x and v there after every iteration of the run.  The averaging
+kernel is checked over all columns (the oracle's averaging is cheap).  The adaptive schedule
+at full size is checked on its first sync interval (oracle over all columns) and by replaying
+Algorithm 2 on the trace the run reports.
+"""
+import numpy as np
+import pytest
+
+from oracle import oracle as O
+from paper_2007_06134_gb300 import abi, inputs
+
+pytestmark = [pytest.mark.gpu, pytest.mark.slow]
+
+torch = pytest.importorskip("torch")
+DEV = "cuda:0"
+REL = 1e-4
+SAMPLE_WIDTH = 1024
+
+
+def _dev(a):
+    return torch.from_numpy(np.ascontiguousarray(a)).to(DEV)
+
+
+def _rel(a, b):
+    return abs(a - b) / max(abs(b), 1e-300)
+
+
+def _sample_ranges(P, count=6):
+    """Disjoint column ranges: the first and last SAMPLE_WIDTH columns and one random range
+    (start a multiple of 4) inside each of `count` equal segments in between."""
+    rng = np.random.default_rng(P)
+    ranges = [(0, SAMPLE_WIDTH)]
+    seg = (P - 2 * SAMPLE_WIDTH) // count
+    for t in range(count):
+        lo = SAMPLE_WIDTH + t * seg
+        start = lo + 4 * int(rng.integers(0, max(1, (seg - SAMPLE_WIDTH) // 4)))
+        ranges.append((start, start + SAMPLE_WIDTH))
+    ranges.append((P - SAMPLE_WIDTH, P))
+    assert all(a[1] <= b[0] for a, b in zip(ranges, ranges[1:]))
+    return ranges
+
+
+def _cfg(w, noise=False):
+    return abi.make_config(w.n, w.P, momentum=w.mu, weight_decay=w.wd, noise_sigma=w.sigma, seed=w.seed,
+                           noise_mode=abi.NOISE_BF16 if noise else abi.NOISE_PHILOX)
+
+
+def _oracle_noise_on_ranges(w, ranges):
+    """The bf16 noise tensor on the sampled columns, from the oracle (zero elsewhere)."""
+    noise = np.zeros((w.n, w.P), np.uint16)
+    for j0, j1 in ranges:
+        for i in range(w.n):
+            noise[i, j0:j1] = O.to_bf16(O.normals(w.seed, 1, i, 0, j0, j1 - j0))
+    return noise
+
+
+@pytest.mark.parametrize("name,p", [("resnet18-n8", 8), ("vgg16-n8", 8), ("resnet50-n16-bf16noise", 4)])
+def test_full_size_constant_period_run_on_sampled_columns(name, p):
+    w = inputs.WORKLOADS[name]
+    bf16 = w.noise == "bf16"
+    h, c = inputs.problem(w)
+    ranges = _sample_ranges(w.P)
+    # GPU: the whole run at full size
+    xd = torch.zeros((w.n, w.P), dtype=torch.float32, device=DEV)
+    vd = torch.zeros_like(xd)
+    nd = None
+    if bf16:
+        nd = torch.empty((w.n, w.P), dtype=torch.int16, device=DEV)
+        abi.adpsgd_noise_fill_bf16(w.seed, w.n, w.P, nd)
+    sched = abi.make_schedule(abi.CPSGD, w.K, p, lr0=w.lr0, lr_factor=w.lr_factor, milestones=w.milestones)
+    tr = abi.TraceBuffers(w.K)
+    with abi.adpsgd_init(_cfg(w, bf16), xd, vd, _dev(h), _dev(c), nd) as ctx:
+        stats = abi.adpsgd_run(ctx, sched, abi.adpsgd_state_init(sched), trace=tr)
+    torch.cuda.synchronize()
+    assert stats.rounds == w.K // p and stats.local_step_launches == w.K
+    # oracle: the same run on the sampled columns only
+    x = np.zeros((w.n, w.P), np.float32)
+    v = np.zeros((w.n, w.P), np.float32)
+    noise = _oracle_noise_on_ranges(w, ranges) if bf16 else None
+    if bf16:
+        for j0, j1 in ranges:
+            gn = nd[:, j0:j1].cpu().numpy().view(np.uint16)
+            assert np.array_equal(gn, noise[:, j0:j1])
+    spec = O.ScheduleSpec(kind=0, K=w.K, p_init=p, lr0=w.lr0, lr_factor=w.lr_factor, milestones=w.milestones)
+    for k in range(w.K):
+        g = O.gamma(spec, k)
+        for j0, j1 in ranges:
+            O.local_step(x, v, h, c, seed=w.seed, k=k, gamma=g, mu=w.mu, wd=w.wd, sigma=w.sigma, noise=noise,
+                         j0=j0, j1=j1)
+        if (k + 1) % p == 0:
+            for j0, j1 in ranges:
+                O.average_variance(x, h, c, j0, j1)
+    for j0, j1 in ranges:
+        gx = xd[:, j0:j1].cpu().numpy()
+        gv = vd[:, j0:j1].cpu().numpy()
+        assert np.array_equal(gx.view(np.uint32), x[:, j0:j1].view(np.uint32)), (name, j0)
+        assert np.array_equal(gv.view(np.uint32), v[:, j0:j1].view(np.uint32)), (name, j0)
+
+
+@pytest.mark.parametrize("name", ["resnet18-n8", "vgg16-n8", "resnet50-n16-bf16noise"])
+def test_full_size_average_and_variance(name):
+    w = inputs.WORKLOADS[name]
+    h, c = inputs.problem(w)
+    x, _ = inputs.random_state(w.n, w.P, 5)
+    xd = _dev(x)
+    with abi.adpsgd_init(_cfg(w), xd, torch.empty_like(xd), _dev(h), _dev(c)) as ctx:
+        D, L = abi.adpsgd_average_and_variance(ctx)
+    torch.cuda.synchronize()
+    Do, Lo = O.average_variance(x, h, c)
+    assert _rel(D, Do) < REL and _rel(L, Lo) < REL
+    got = xd.cpu().numpy()
+    assert np.array_equal(got.view(np.uint32), x.view(np.uint32))
+
+
+def test_full_size_adaptive_first_interval_and_rule_replay():
+    # resnet18-n8 at full size, Algorithm 2 (p_init 4, K_s 500): the first sync (after 4 local
+    # steps from x0 = 0) against the oracle over all columns, and the whole trace against
+    # Algorithm 2 replayed on the S values the run reported.
+    w = inputs.WORKLOADS["resnet18-n8"]
+    h, c = inputs.problem(w)
+    xd = torch.zeros((w.n, w.P), dtype=torch.float32, device=DEV)
+    vd = torch.zeros_like(xd)
+    sched = abi.make_schedule(abi.ADPSGD, w.K, w.p_init, K_s=w.K_s, lr0=w.lr0, lr_factor=w.lr_factor,
+                              milestones=w.milestones)
+    tr = abi.TraceBuffers(w.K)
+    with abi.adpsgd_init(_cfg(w), xd, vd, _dev(h), _dev(c)) as ctx:
+        stats = abi.adpsgd_run(ctx, sched, abi.adpsgd_state_init(sched), trace=tr)
+    t = tr.arrays()
+    assert stats.rounds == len(t["k"]) and t["k"][0] == w.p_init - 1
+
+    x, v = inputs.zero_state(w.n, w.P)
+    for k in range(w.p_init):
+        O.local_step(x, v, h, c, seed=w.seed, k=k, gamma=np.float32(w.lr0), mu=w.mu, wd=w.wd, sigma=w.sigma)
+    D0, L0 = O.average_variance(x, h, c)
+    assert _rel(t["S"][0], D0 / w.n) < REL and _rel(t["loss"][0], L0) < REL
+
+    spec = O.ScheduleSpec(kind=1, K=w.K, p_init=w.p_init, K_s=w.K_s, lr0=w.lr0, lr_factor=w.lr_factor,
+                          milestones=w.milestones)
+    st = O.new_state(spec)
+    k_expect = w.p_init - 1
+    for s in range(len(t["k"])):
+        assert t["k"][s] == k_expect
+        O.on_sync(spec, st, int(t["k"][s]), float(t["S"][s]), O.gamma(spec, int(t["k"][s])))
+        assert t["p"][s] == st.p and t["C2"][s] == st.C2
+        k_expect += st.p
+    assert k_expect >= w.K
