@@ -308,6 +308,7 @@ def run_gpu(args, w):
     value = world * rp_per_step / (ms_step / 1000.0)
 
     kt = abi.adpsgd_kernel_times(ctx)
+    kt = dict(kt)
     peak, peak_kind = measured_peaks()
     k1_bytes = 16 * n * P + 8 * P + (2 * n * P if noise is not None else 0)
     k1_ms = kt["local_step_ms"] / max(1, kt["local_step_launches"])
@@ -351,6 +352,33 @@ def run_gpu(args, w):
         e2e_value = world * rp_per_step / dt
         ctx_e2e.close()
 
+    # The same run with each sync interval fused into one kernel (separable objective only).
+    fused = None
+    if not args.no_fused and n <= 32:
+        cfg_f = abi.make_config(n, P, momentum=w.mu, weight_decay=w.wd, noise_sigma=w.sigma, seed=seed,
+                                noise_mode=cfg.noise_mode, want_loss=True, time_kernels=True, fuse_intervals=True)
+        with abi.adpsgd_init(cfg_f, xd, vd, hd, cd, noise, stream) as ctx_f:
+            def fused_run():
+                xd.zero_()
+                vd.zero_()
+                return abi.adpsgd_run(ctx_f, sched, abi.adpsgd_state_init(sched))
+            fused_run()
+            abi.adpsgd_reset_kernel_times(ctx_f)
+            torch.cuda.synchronize(device)
+            barrier(pg, device)
+            ev0.record(stream)
+            for _ in range(args.steps):
+                fstats = fused_run()
+            ev1.record(stream)
+            torch.cuda.synchronize(device)
+            fms = max_over_ranks(pg, ev0.elapsed_time(ev1), device) / args.steps
+            ft = abi.adpsgd_kernel_times(ctx_f)
+        fused = {"value": world * rp_per_step / (fms / 1000.0), "unit": UNIT, "ms_per_step": fms,
+                 "interval_launches_per_step": fstats.interval_launches,
+                 "interval_ms_per_launch": ft["interval_ms"] / max(1, ft["interval_launches"]),
+                 "note": "each sync interval (local steps + averaging) as one kernel; valid for the "
+                         "separable surrogate objective only, not for a real model"}
+
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu:
         r, dt, sample = oracle_sample(w)
@@ -377,6 +405,7 @@ def run_gpu(args, w):
                              "ms_per_launch": k2_ms, "launches": kt["average_launches"],
                              "traffic": recorded_traffic("average_kernel", w.name)},
             "local_step_rp_per_s": n * P / (k1_ms / 1000.0),
+            "fused_intervals": fused,
             "clocks": clock_summary,
             "cpu_baseline": cpu,
         }
@@ -433,6 +462,7 @@ def main():
                     help="override the workload's iteration count (profiling captures only)")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu", action="store_true")
+    ap.add_argument("--no-fused", action="store_true", help="skip the fused-interval measurement")
     ap.add_argument("--sweep", action="store_true", help="averaging-kernel sweep over n x P instead")
     ap.add_argument("--sweep-max-bytes", type=float, default=70e9)
     args = ap.parse_args()

@@ -65,7 +65,11 @@ typedef struct {
     uint64_t seed;           /* Philox key (low word, high word) */
     int64_t wait_timeout_ms; /* bound on every host wait; <= 0 means 60000 */
     int32_t time_kernels;    /* nonzero: bracket every kernel launch with CUDA events */
-    int32_t reserved;
+    int32_t fuse_intervals;  /* nonzero (needs n <= 32): adpsgd_run and adpsgd_local_steps run each
+                                stretch of local steps up to the next sync (at most 256 steps), and
+                                the sync's averaging, as ONE kernel that keeps x and v in registers
+                                between steps.  Results are bit-identical to the unfused path.  Valid
+                                only because the surrogate objective is separable per column. */
 } adpsgd_config;
 
 /* Schedules (Algorithm 1: kind 0; Algorithm 2: kind 1). */
@@ -117,15 +121,27 @@ typedef struct {
     double wire_bytes_per_node;      /* ring allreduce of P fp32 + one fp32 S_k, per sync */
     double wire_bytes_total;         /* times n */
     double fullsgd_wire_bytes_per_node; /* one P-fp32 allreduce per iteration (FULLSGD) */
-    int64_t local_step_launches;     /* kernel launches issued by this call */
-    int64_t average_launches;
+    int64_t local_step_launches;     /* kernel launches issued by this call: local steps, */
+    int64_t average_launches;        /* averagings, */
+    int64_t interval_launches;       /* and fused intervals (cfg.fuse_intervals) */
 } adpsgd_stats;
+
+/* Device time of the kernels launched through a context, from CUDA events on its stream. */
+typedef struct {
+    double local_step_ms;
+    int64_t local_step_launches;
+    double average_ms;
+    int64_t average_launches;
+    double interval_ms;
+    int64_t interval_launches;
+} adpsgd_kernel_timing;
 
 /* Create a context over caller-owned device arrays.
  * x, v: [n, P] fp32 (read/write); h, c: [P] fp32 (read only);
  * noise_bf16: [n, P] bf16 (read only) when cfg->noise_mode == ADPSGD_NOISE_BF16, else NULL.
  * The pointers must stay valid until adpsgd_destroy.  Errors: E_INVAL (bad n, P, NULL
- * pointer, P*n overflow), E_ALIGN, E_NOMEM, E_CUDA.  On error *out is NULL. */
+ * pointer, P*n overflow, fuse_intervals with n > 32), E_ALIGN, E_NOMEM, E_CUDA.  On error
+ * *out is NULL. */
 int adpsgd_init(const adpsgd_config* cfg, float* x, float* v, const float* h, const float* c,
                 const uint16_t* noise_bf16, void* stream, adpsgd_ctx** out);
 
@@ -222,9 +238,8 @@ int adpsgd_noise_fill_bf16(uint64_t seed, int32_t n, int64_t P, uint16_t* out, v
 
 /* Device time of the kernels launched through ctx while cfg.time_kernels was set, summed from
  * CUDA events on ctx's stream since init or the last reset (waits for them, bounded).
- * Any output pointer may be NULL.  Errors: E_STATE (timing off), E_TIMEOUT, E_CUDA. */
-int adpsgd_kernel_times(adpsgd_ctx* ctx, double* local_step_ms, int64_t* local_step_launches,
-                        double* average_ms, int64_t* average_launches);
+ * Errors: E_INVAL (out NULL), E_STATE (timing off), E_TIMEOUT, E_CUDA. */
+int adpsgd_kernel_times(adpsgd_ctx* ctx, adpsgd_kernel_timing* out);
 int adpsgd_reset_kernel_times(adpsgd_ctx* ctx);
 
 /* Test hook: when force_incomplete is nonzero every bounded wait of ctx behaves as if the

@@ -34,7 +34,7 @@ class Config(C.Structure):
     _fields_ = [("n", C.c_int32), ("noise_mode", C.c_int32), ("P", C.c_int64), ("momentum", C.c_float),
                 ("weight_decay", C.c_float), ("noise_sigma", C.c_float), ("want_loss", C.c_int32),
                 ("seed", C.c_uint64), ("wait_timeout_ms", C.c_int64), ("time_kernels", C.c_int32),
-                ("reserved", C.c_int32)]
+                ("fuse_intervals", C.c_int32)]
 
 
 class Schedule(C.Structure):
@@ -59,7 +59,13 @@ class Trace(C.Structure):
 class Stats(C.Structure):
     _fields_ = [("rounds", C.c_int64), ("equiv_period", C.c_double), ("wire_bytes_per_node", C.c_double),
                 ("wire_bytes_total", C.c_double), ("fullsgd_wire_bytes_per_node", C.c_double),
-                ("local_step_launches", C.c_int64), ("average_launches", C.c_int64)]
+                ("local_step_launches", C.c_int64), ("average_launches", C.c_int64),
+                ("interval_launches", C.c_int64)]
+
+
+class KernelTiming(C.Structure):
+    _fields_ = [("local_step_ms", C.c_double), ("local_step_launches", C.c_int64), ("average_ms", C.c_double),
+                ("average_launches", C.c_int64), ("interval_ms", C.c_double), ("interval_launches", C.c_int64)]
 
 
 _P = C.c_void_p
@@ -81,8 +87,7 @@ _SIGS = {
     "adpsgd_philox_fill": (C.c_int, [C.c_uint64, C.c_uint32, C.c_int32, C.c_int64, C.c_int64, _P, _P]),
     "adpsgd_noise_fill_f32": (C.c_int, [C.c_uint64, C.c_uint32, C.c_int32, C.c_int64, C.c_int64, _P, _P]),
     "adpsgd_noise_fill_bf16": (C.c_int, [C.c_uint64, C.c_int32, C.c_int64, _P, _P]),
-    "adpsgd_kernel_times": (C.c_int, [_P, C.POINTER(C.c_double), C.POINTER(C.c_int64), C.POINTER(C.c_double),
-                                      C.POINTER(C.c_int64)]),
+    "adpsgd_kernel_times": (C.c_int, [_P, C.POINTER(KernelTiming)]),
     "adpsgd_reset_kernel_times": (C.c_int, [_P]),
     "adpsgd_test_force_incomplete": (C.c_int, [_P, C.c_int32]),
     "adpsgd_destroy": (None, [_P]),
@@ -151,9 +156,9 @@ def _stream(stream) -> int | None:
 
 
 def make_config(n, P, *, momentum=0.9, weight_decay=0.0, noise_sigma=1.0, seed=0, noise_mode=NOISE_PHILOX,
-                want_loss=True, wait_timeout_ms=60000, time_kernels=False) -> Config:
+                want_loss=True, wait_timeout_ms=60000, time_kernels=False, fuse_intervals=False) -> Config:
     return Config(n, noise_mode, P, momentum, weight_decay, noise_sigma, int(bool(want_loss)),
-                  seed & 0xFFFFFFFFFFFFFFFF, wait_timeout_ms, int(bool(time_kernels)), 0)
+                  seed & 0xFFFFFFFFFFFFFFFF, wait_timeout_ms, int(bool(time_kernels)), int(bool(fuse_intervals)))
 
 
 def make_schedule(kind, K, p_init, *, K_s=0, K_w=0, lo=0.7, hi=1.3, p_min=1, p_max=0, lr0=0.1, lr_factor=0.1,
@@ -308,12 +313,9 @@ def adpsgd_noise_fill_bf16(seed: int, n: int, P: int, out, stream=None) -> None:
 
 
 def adpsgd_kernel_times(ctx: Context):
-    a, c = C.c_double(), C.c_double()
-    b, d = C.c_int64(), C.c_int64()
-    _check(load().adpsgd_kernel_times(ctx.handle, C.byref(a), C.byref(b), C.byref(c), C.byref(d)),
-           "adpsgd_kernel_times")
-    return dict(local_step_ms=a.value, local_step_launches=b.value, average_ms=c.value,
-                average_launches=d.value)
+    t = KernelTiming()
+    _check(load().adpsgd_kernel_times(ctx.handle, C.byref(t)), "adpsgd_kernel_times")
+    return {name: getattr(t, name) for name, _ in KernelTiming._fields_}
 
 
 def adpsgd_reset_kernel_times(ctx: Context) -> None:

@@ -1,9 +1,9 @@
 """Build ``libadpsgd.so`` (the C ABI of include/adpsgd.h) in-tree for sm_103a.
 
-kernels.cu is compiled by nvcc for sm_103a only, with IEEE division and square root,
-no flush-to-zero and no multiply-add contraction (the generator and the update are
-specified operation by operation); runtime.cpp is host C++.  The two objects are
-compiled in parallel and linked by nvcc with the static CUDA runtime.
+Every .cu file in csrc/ is compiled by nvcc for sm_103a only, with IEEE division and square
+root, no flush-to-zero and no multiply-add contraction (the generator and the update are
+specified operation by operation); every .cpp file is host C++.  The objects are compiled in
+parallel and linked by nvcc with the static CUDA runtime.
 """
 from __future__ import annotations
 
@@ -63,23 +63,31 @@ def build(force: bool = False, verbose: bool = False) -> str:
     cuda = _cuda_home()
     nvcc = os.path.join(cuda, "bin", "nvcc")
     os.makedirs(BUILD, exist_ok=True)
-    k_obj = os.path.join(BUILD, "kernels.o")
-    r_obj = os.path.join(BUILD, "runtime.o")
-    jobs = [
-        ([nvcc, *ARCH, *NVCC_FLAGS, "-I", INCLUDE, "-c", os.path.join(CSRC, "kernels.cu"), "-o", k_obj],
-         os.path.join(BUILD, "kernels.log")),
-        (["g++", *CXX_FLAGS, "-I", os.path.join(cuda, "include"), "-I", INCLUDE, "-c",
-          os.path.join(CSRC, "runtime.cpp"), "-o", r_obj], os.path.join(BUILD, "runtime.log")),
-    ]
-    with ThreadPoolExecutor(2) as ex:
-        for f in [ex.submit(_run, c, l) for c, l in jobs]:
-            f.result()
+    jobs, objs = [], []
+    for f in sorted(os.listdir(CSRC)):
+        src = os.path.join(CSRC, f)
+        stem, ext = os.path.splitext(f)
+        obj = os.path.join(BUILD, stem + ".o")
+        if ext == ".cu":
+            jobs.append(([nvcc, *ARCH, *NVCC_FLAGS, "-I", INCLUDE, "-c", src, "-o", obj],
+                         os.path.join(BUILD, stem + ".log")))
+        elif ext == ".cpp":
+            jobs.append((["g++", *CXX_FLAGS, "-I", os.path.join(cuda, "include"), "-I", INCLUDE, "-c", src, "-o", obj],
+                         os.path.join(BUILD, stem + ".log")))
+        else:
+            continue
+        objs.append(obj)
+    with ThreadPoolExecutor(len(jobs)) as ex:
+        for fut in [ex.submit(_run, c, l) for c, l in jobs]:
+            fut.result()
     tmp = LIB + f".tmp{os.getpid()}"
-    _run([nvcc, *ARCH, "-shared", "-o", tmp, k_obj, r_obj, "-cudart", "static"], os.path.join(BUILD, "link.log"))
+    _run([nvcc, *ARCH, "-shared", "-o", tmp, *objs, "-cudart", "static"], os.path.join(BUILD, "link.log"))
     os.replace(tmp, LIB)
     if verbose:
-        with open(os.path.join(BUILD, "kernels.log")) as f:
-            sys.stdout.write(f.read())
+        for f in sorted(os.listdir(BUILD)):
+            if f.endswith(".log") and f != "link.log":
+                with open(os.path.join(BUILD, f)) as fh:
+                    sys.stdout.write(fh.read())
     return LIB
 
 

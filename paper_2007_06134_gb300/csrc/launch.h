@@ -57,6 +57,34 @@ int average_grid_max(int sms);
 int static_scratch_max_blocks();
 cudaError_t static_scratch_address(double** partials, double** out, unsigned int** counter);
 
+// A fused sync interval: m (<= kMaxFusedSteps) local steps of every replica from step k0 with
+// step sizes gamma[0..m), then (average) the averaging with its sums in out[0..1].  n <= 32.
+constexpr int kMaxFusedSteps = 256;
+struct IntervalArgs {
+    float* x;
+    float* v;
+    const float* h;
+    const float* c;
+    const uint16_t* noise_bf16;
+    const PhiloxKeys* keys;
+    int32_t n;
+    int64_t P;
+    uint32_t k0;
+    int32_t m;
+    const float* gamma;  // host array of m step sizes
+    float mu, wd, sigma;
+    bool average;
+    bool loss;
+    double* partials;  // 2 * grid
+    double* out;
+    unsigned int* counter;
+    int grid;  // from interval_grid()
+};
+cudaError_t launch_interval(const IntervalArgs& a, cudaStream_t stream);
+int interval_grid(int32_t n, int64_t P, int sms);
+int interval_grid_max(int sms);
+int interval_max_replicas();
+
 cudaError_t launch_philox_fill(uint64_t seed, uint32_t tag, int32_t n, int64_t nq, uint32_t k,
                                uint32_t* out, cudaStream_t stream);
 cudaError_t launch_noise_f32(uint64_t seed, uint32_t tag, int32_t n, int64_t P, uint32_t k,

@@ -3,6 +3,7 @@
 // waits.  All device work goes through the kernels in kernels.cu on the caller's stream.
 #include <cuda_runtime_api.h>
 
+#include <algorithm>
 #include <chrono>
 #include <cstdint>
 #include <cstdio>
@@ -33,7 +34,7 @@ constexpr int64_t kMaxK = int64_t(1) << 32;  // the step index is one 32-bit Phi
 
 struct TimedLaunch {
     cudaEvent_t start, stop;
-    int kind;  // 0 local step, 1 averaging
+    int kind;  // 0 local step, 1 averaging, 2 fused interval
 };
 
 struct adpsgd_ctx {
@@ -51,13 +52,13 @@ struct adpsgd_ctx {
     double* d_out = nullptr;  // D, loss, then the averaging kernel's completion counter
     double* h_out = nullptr;  // pinned, 2 doubles
     cudaEvent_t done = nullptr;
-    int grid_avg = 0, grid_avg_loss = 0, grid_var = 0;
+    int grid_avg = 0, grid_avg_loss = 0, grid_var = 0, grid_interval = 0;
     // kernel timing
     std::vector<cudaEvent_t> free_events;
     std::vector<TimedLaunch> pending;
-    double ms[2] = {0.0, 0.0};
-    int64_t launches[2] = {0, 0};
-    int64_t timed_launches[2] = {0, 0};
+    double ms[3] = {0.0, 0.0, 0.0};
+    int64_t launches[3] = {0, 0, 0};
+    int64_t timed_launches[3] = {0, 0, 0};
     bool force_incomplete = false;
 };
 
@@ -194,6 +195,41 @@ int average(adpsgd_ctx* ctx, bool write_back, bool loss)
     return wait_event(ctx, ctx->done);
 }
 
+// Enqueue one fused interval: m local steps from step k0 (step sizes gamma[0..m)) and, if
+// `average`, the averaging with the copy of its sums and ctx->done.
+int interval(adpsgd_ctx* ctx, int64_t k0, int32_t m, const float* gamma, bool average, bool loss)
+{
+    adpsgd::IntervalArgs a;
+    a.x = ctx->x;
+    a.v = ctx->v;
+    a.h = ctx->h;
+    a.c = ctx->c;
+    a.noise_bf16 = ctx->cfg.noise_mode == ADPSGD_NOISE_BF16 ? ctx->noise : nullptr;
+    a.keys = &ctx->keys;
+    a.n = ctx->cfg.n;
+    a.P = ctx->cfg.P;
+    a.k0 = (uint32_t)k0;
+    a.m = m;
+    a.gamma = gamma;
+    a.mu = ctx->cfg.momentum;
+    a.wd = ctx->cfg.weight_decay;
+    a.sigma = ctx->cfg.noise_sigma;
+    a.average = average;
+    a.loss = average && loss;
+    a.partials = ctx->d_partials;
+    a.out = ctx->d_out;
+    a.counter = reinterpret_cast<unsigned int*>(ctx->d_out + 2);
+    a.grid = ctx->grid_interval;
+    int st = timed(ctx, 2, [&] { return adpsgd::launch_interval(a, ctx->stream); }, "interval");
+    if (st != ADPSGD_OK || !average) return st;
+    cudaError_t e = cudaMemcpyAsync(ctx->h_out, ctx->d_out, 2 * sizeof(double), cudaMemcpyDeviceToHost,
+                                    ctx->stream);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaMemcpyAsync");
+    e = cudaEventRecord(ctx->done, ctx->stream);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaEventRecord");
+    return ADPSGD_OK;
+}
+
 int check_schedule(const adpsgd_schedule* s)
 {
     if (s == nullptr) return ADPSGD_E_INVAL;
@@ -293,6 +329,7 @@ int adpsgd_init(const adpsgd_config* cfg, float* x, float* v, const float* h, co
     if (cfg->noise_mode == ADPSGD_NOISE_BF16 && noise_bf16 == nullptr) return ADPSGD_E_INVAL;
     if (!aligned16(x) || !aligned16(v) || !aligned16(h) || !aligned16(c)) return ADPSGD_E_ALIGN;
     if (noise_bf16 != nullptr && !aligned16(noise_bf16)) return ADPSGD_E_ALIGN;
+    if (cfg->fuse_intervals && cfg->n > adpsgd::interval_max_replicas()) return ADPSGD_E_INVAL;
 
     adpsgd_ctx* ctx = new (std::nothrow) adpsgd_ctx();
     if (ctx == nullptr) return ADPSGD_E_NOMEM;
@@ -314,7 +351,9 @@ int adpsgd_init(const adpsgd_config* cfg, float* x, float* v, const float* h, co
     ctx->grid_avg = adpsgd::average_grid(cfg->n, cfg->P, false, true, ctx->sms);
     ctx->grid_avg_loss = adpsgd::average_grid(cfg->n, cfg->P, true, true, ctx->sms);
     ctx->grid_var = adpsgd::average_grid(cfg->n, cfg->P, false, false, ctx->sms);
-    const size_t partial_bytes = 2 * sizeof(double) * (size_t)adpsgd::average_grid_max(ctx->sms);
+    if (cfg->fuse_intervals) ctx->grid_interval = adpsgd::interval_grid(cfg->n, cfg->P, ctx->sms);
+    const int max_grid = std::max(adpsgd::average_grid_max(ctx->sms), adpsgd::interval_grid_max(ctx->sms));
+    const size_t partial_bytes = 2 * sizeof(double) * (size_t)max_grid;
     e = cudaMalloc(reinterpret_cast<void**>(&ctx->d_partials), partial_bytes);
     if (e == cudaSuccess) e = cudaMalloc(reinterpret_cast<void**>(&ctx->d_out), 4 * sizeof(double));
     if (e == cudaSuccess) e = cudaMemset(ctx->d_out, 0, 4 * sizeof(double));
@@ -354,6 +393,14 @@ void adpsgd_destroy(adpsgd_ctx* ctx)
 int adpsgd_local_steps(adpsgd_ctx* ctx, int64_t k0, int32_t m, const float* lr)
 {
     if (ctx == nullptr || m < 0 || k0 < 0 || k0 + m > kMaxK || (m > 0 && lr == nullptr)) return ADPSGD_E_INVAL;
+    if (ctx->cfg.fuse_intervals) {
+        for (int32_t t = 0; t < m; t += adpsgd::kMaxFusedSteps) {
+            const int32_t chunk = std::min<int32_t>(adpsgd::kMaxFusedSteps, m - t);
+            int st = interval(ctx, k0 + t, chunk, lr + t, false, false);
+            if (st != ADPSGD_OK) return st;
+        }
+        return ADPSGD_OK;
+    }
     for (int32_t t = 0; t < m; ++t) {
         int st = local_step(ctx, k0 + t, lr[t]);
         if (st != ADPSGD_OK) return st;
@@ -431,7 +478,49 @@ int adpsgd_run(adpsgd_ctx* ctx, const adpsgd_schedule* sched, adpsgd_state* stat
     const bool loss = ctx->cfg.want_loss != 0;
     const int64_t stop = k_end < sched->K ? k_end : sched->K;
     const int64_t launches0[2] = {ctx->launches[0], ctx->launches[1]};
+    const int64_t launches_fused0 = ctx->launches[2];
     bool launched_ahead = false;  // the local step of iteration k is already enqueued
+    if (ctx->cfg.fuse_intervals) {
+        // One kernel per stretch of iterations up to and including the next sync (at most
+        // kMaxFusedSteps); sync_after advances cnt exactly as in the unfused loop below.
+        float gam[adpsgd::kMaxFusedSteps];
+        int64_t k = state->k_next;
+        while (k < stop) {
+            int32_t m = 0;
+            bool sync = false;
+            while (k + m < stop && m < adpsgd::kMaxFusedSteps) {
+                gam[m] = gamma_of(sched, k + m);
+                const bool s_now = sync_after(sched, state, k + m);
+                ++m;
+                if (s_now) {
+                    sync = true;
+                    break;
+                }
+            }
+            st = interval(ctx, k, m, gam, sync, loss);
+            if (st != ADPSGD_OK) return st;
+            state->k_next = k + m;
+            if (sync) {
+                st = wait_event(ctx, ctx->done);
+                if (st != ADPSGD_OK) return st;
+                const int64_t ks = k + m - 1;
+                const double S = ctx->h_out[0] / (double)ctx->cfg.n;
+                const int32_t phase = rule(sched, state, ks, S, (double)gam[m - 1]);
+                if (trace != nullptr && trace->len < trace->cap) {
+                    const int64_t t = trace->len;
+                    trace->k[t] = ks;
+                    trace->p[t] = state->p;
+                    trace->S[t] = S;
+                    trace->C2[t] = state->C2;
+                    trace->loss[t] = loss ? ctx->h_out[1] : 0.0;
+                    trace->phase[t] = phase;
+                    trace->len = t + 1;
+                }
+                state->rounds += 1;
+            }
+            k += m;
+        }
+    }
     for (int64_t k = state->k_next; k < stop; ++k) {
         if (!launched_ahead) {
             st = local_step(ctx, k, gamma_of(sched, k));
@@ -476,6 +565,7 @@ int adpsgd_run(adpsgd_ctx* ctx, const adpsgd_schedule* sched, adpsgd_state* stat
         wire(ctx->cfg.n, ctx->cfg.P, state->k_next, false, &stats->fullsgd_wire_bytes_per_node, &total);
         stats->local_step_launches = ctx->launches[0] - launches0[0];
         stats->average_launches = ctx->launches[1] - launches0[1];
+        stats->interval_launches = ctx->launches[2] - launches_fused0;
     }
     return ADPSGD_OK;
 }
@@ -561,17 +651,18 @@ int adpsgd_noise_fill_bf16(uint64_t seed, int32_t n, int64_t P, uint16_t* out, v
     return e == cudaSuccess ? ADPSGD_OK : cuda_fail(e, "bf16 noise fill");
 }
 
-int adpsgd_kernel_times(adpsgd_ctx* ctx, double* local_step_ms, int64_t* local_step_launches, double* average_ms,
-                        int64_t* average_launches)
+int adpsgd_kernel_times(adpsgd_ctx* ctx, adpsgd_kernel_timing* out)
 {
-    if (ctx == nullptr) return ADPSGD_E_INVAL;
+    if (ctx == nullptr || out == nullptr) return ADPSGD_E_INVAL;
     if (!ctx->cfg.time_kernels) return ADPSGD_E_STATE;
     int st = harvest_times(ctx);
     if (st != ADPSGD_OK) return st;
-    if (local_step_ms != nullptr) *local_step_ms = ctx->ms[0];
-    if (local_step_launches != nullptr) *local_step_launches = ctx->timed_launches[0];
-    if (average_ms != nullptr) *average_ms = ctx->ms[1];
-    if (average_launches != nullptr) *average_launches = ctx->timed_launches[1];
+    out->local_step_ms = ctx->ms[0];
+    out->local_step_launches = ctx->timed_launches[0];
+    out->average_ms = ctx->ms[1];
+    out->average_launches = ctx->timed_launches[1];
+    out->interval_ms = ctx->ms[2];
+    out->interval_launches = ctx->timed_launches[2];
     return ADPSGD_OK;
 }
 
@@ -582,8 +673,8 @@ int adpsgd_reset_kernel_times(adpsgd_ctx* ctx)
         int st = harvest_times(ctx);
         if (st != ADPSGD_OK) return st;
     }
-    ctx->ms[0] = ctx->ms[1] = 0.0;
-    ctx->timed_launches[0] = ctx->timed_launches[1] = 0;
+    ctx->ms[0] = ctx->ms[1] = ctx->ms[2] = 0.0;
+    ctx->timed_launches[0] = ctx->timed_launches[1] = ctx->timed_launches[2] = 0;
     return ADPSGD_OK;
 }
 

@@ -44,9 +44,9 @@ def _sample_ranges(P, count=6):
     return ranges
 
 
-def _cfg(w, noise=False):
+def _cfg(w, noise=False, fused=False):
     return abi.make_config(w.n, w.P, momentum=w.mu, weight_decay=w.wd, noise_sigma=w.sigma, seed=w.seed,
-                           noise_mode=abi.NOISE_BF16 if noise else abi.NOISE_PHILOX)
+                           noise_mode=abi.NOISE_BF16 if noise else abi.NOISE_PHILOX, fuse_intervals=fused)
 
 
 def _oracle_noise_on_ranges(w, ranges):
@@ -58,8 +58,10 @@ def _oracle_noise_on_ranges(w, ranges):
     return noise
 
 
-@pytest.mark.parametrize("name,p", [("resnet18-n8", 8), ("vgg16-n8", 8), ("resnet50-n16-bf16noise", 4)])
-def test_full_size_constant_period_run_on_sampled_columns(name, p):
+@pytest.mark.parametrize("name,p,fused", [("resnet18-n8", 8, False), ("vgg16-n8", 8, False),
+                                          ("resnet50-n16-bf16noise", 4, False), ("resnet18-n8", 8, True),
+                                          ("resnet50-n16-bf16noise", 4, True)])
+def test_full_size_constant_period_run_on_sampled_columns(name, p, fused):
     w = inputs.WORKLOADS[name]
     bf16 = w.noise == "bf16"
     h, c = inputs.problem(w)
@@ -73,10 +75,11 @@ def test_full_size_constant_period_run_on_sampled_columns(name, p):
         abi.adpsgd_noise_fill_bf16(w.seed, w.n, w.P, nd)
     sched = abi.make_schedule(abi.CPSGD, w.K, p, lr0=w.lr0, lr_factor=w.lr_factor, milestones=w.milestones)
     tr = abi.TraceBuffers(w.K)
-    with abi.adpsgd_init(_cfg(w, bf16), xd, vd, _dev(h), _dev(c), nd) as ctx:
+    with abi.adpsgd_init(_cfg(w, bf16, fused), xd, vd, _dev(h), _dev(c), nd) as ctx:
         stats = abi.adpsgd_run(ctx, sched, abi.adpsgd_state_init(sched), trace=tr)
     torch.cuda.synchronize()
-    assert stats.rounds == w.K // p and stats.local_step_launches == w.K
+    assert stats.rounds == w.K // p
+    assert (stats.interval_launches if fused else stats.local_step_launches) == (w.K // p if fused else w.K)
     # oracle: the same run on the sampled columns only
     x = np.zeros((w.n, w.P), np.float32)
     v = np.zeros((w.n, w.P), np.float32)
