@@ -451,6 +451,64 @@ def run_sweep(args):
             del xd
 
 
+def run_variance_traces(args):
+    """The schedule study of Sec. IV on the strategies-n16 surrogate: constant periods, the four
+    strategies' piecewise periods, the decreasing period of Sec. VI-B and Algorithm 2, each a whole
+    run with Var[W_k] recorded every iteration.  One JSON line per schedule: syncs, the weighted
+    variance of Eq. metric2, the mean variance per step-size phase, the loss, and the period."""
+    import torch
+
+    from paper_2007_06134_gb300 import abi, diagnostics, inputs
+    w = inputs.WORKLOADS["strategies-n16"]
+    n, P, K = w.n, w.P, w.K
+    device = torch.device("cuda", 0)
+    stream = torch.cuda.current_stream(device)
+    h, c = inputs.problem(w)
+    hd, cd = torch.from_numpy(h).to(device), torch.from_numpy(c).to(device)
+    xd = torch.zeros((n, P), dtype=torch.float32, device=device)
+    vd = torch.zeros_like(xd)
+    kw = dict(lr0=w.lr0, lr_factor=w.lr_factor, milestones=w.milestones)
+    half = K // 2
+    schedules = [
+        ("FULLSGD (p=1)", abi.make_schedule(abi.CPSGD, K, 1, **kw)),
+        ("CPSGD p=2", abi.make_schedule(abi.CPSGD, K, 2, **kw)),
+        ("CPSGD p=4", abi.make_schedule(abi.CPSGD, K, 4, **kw)),
+        ("CPSGD p=5 (strategy 4)", abi.make_schedule(abi.CPSGD, K, 5, **kw)),
+        ("CPSGD p=8 (strategy 3)", abi.make_schedule(abi.CPSGD, K, 8, **kw)),
+        ("strategy 1: p=4 then 8", abi.make_schedule(abi.PIECEWISE, K, 4, period_changes=((half, 8),), **kw)),
+        ("strategy 2: p=8 then 4", abi.make_schedule(abi.PIECEWISE, K, 8, period_changes=((half, 4),), **kw)),
+        ("decreasing: p=20 then 5", abi.make_schedule(abi.PIECEWISE, K, 20, period_changes=((half, 5),), **kw)),
+        ("ADPSGD p_init=4 K_s=1000 K_w=25", abi.make_schedule(abi.ADPSGD, K, 4, K_s=1000, K_w=25, **kw)),
+    ]
+    gammas = [abi.adpsgd_gamma(schedules[0][1], k) for k in range(K)]
+    edges = [0] + list(w.milestones) + [K]
+    cfg = abi.make_config(n, P, momentum=w.mu, weight_decay=w.wd, noise_sigma=w.sigma, seed=w.seed, want_loss=True)
+    with abi.adpsgd_init(cfg, xd, vd, hd, cd, None, stream) as ctx:
+        for name, sched in schedules:
+            xd.zero_()
+            vd.zero_()
+            tr = abi.TraceBuffers(K + 1, var_cap=K)
+            t0 = time.perf_counter()
+            stats = abi.adpsgd_run(ctx, sched, abi.adpsgd_state_init(sched), trace=tr)
+            dt = time.perf_counter() - t0
+            t = tr.arrays()
+            line = {"variance_traces": w.name, "schedule": name, "syncs": int(stats.rounds),
+                    "equiv_period": K / stats.rounds,
+                    "weighted_variance_eq_metric2": diagnostics.weighted_variance(t["var"], gammas),
+                    "mean_variance_per_lr_phase": diagnostics.phase_means(t["var"], edges),
+                    "mean_V_t": float(np.mean(diagnostics.interval_means(t["var"], t["k"]))),
+                    "final_loss": float(t["loss"][-1]), "min_loss": float(np.min(t["loss"])),
+                    "wire_bytes_per_node": stats.wire_bytes_per_node, "seconds": dt}
+            if sched.kind == abi.ADPSGD:
+                pk = {}
+                for q in (999, 1999, 2999, K - 1):
+                    idx = int(np.searchsorted(t["k"], q, side="right")) - 1
+                    pk[str(q + 1)] = int(t["p"][max(idx, 0)])
+                line["period_at_iteration"] = pk
+                line["C2"] = float(t["C2"][-1])
+            print(json.dumps(line), flush=True)
+
+
 def main():
     ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
     ap.add_argument("--gpus", type=int, default=1)
@@ -465,6 +523,8 @@ def main():
     ap.add_argument("--no-fused", action="store_true", help="skip the fused-interval measurement")
     ap.add_argument("--sweep", action="store_true", help="averaging-kernel sweep over n x P instead")
     ap.add_argument("--sweep-max-bytes", type=float, default=70e9)
+    ap.add_argument("--variance-traces", action="store_true",
+                    help="the schedule study of Sec. IV with per-iteration variance instead")
     args = ap.parse_args()
     from paper_2007_06134_gb300 import inputs
     w = inputs.WORKLOADS[args.workload]
@@ -476,6 +536,8 @@ def main():
         return run_reference(args, w)
     if args.sweep:
         return run_sweep(args)
+    if args.variance_traces:
+        return run_variance_traces(args)
     return run_gpu(args, w)
 
 

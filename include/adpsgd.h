@@ -72,11 +72,12 @@ typedef struct {
                                 only because the surrogate objective is separable per column. */
 } adpsgd_config;
 
-/* Schedules (Algorithm 1: kind 0; Algorithm 2: kind 1). */
-enum { ADPSGD_CPSGD = 0, ADPSGD_ADPSGD = 1 };
+/* Schedules (Algorithm 1: kind 0; Algorithm 2: kind 1; kind 2: a piecewise-constant period,
+ * such as the four strategies of Sec. IV-A and the decreasing period of Sec. VI-B). */
+enum { ADPSGD_CPSGD = 0, ADPSGD_ADPSGD = 1, ADPSGD_PIECEWISE = 2 };
 
 typedef struct {
-    int32_t kind;            /* ADPSGD_CPSGD (constant p) or ADPSGD_ADPSGD */
+    int32_t kind;            /* ADPSGD_CPSGD (constant p), ADPSGD_ADPSGD or ADPSGD_PIECEWISE */
     int32_t p_init;          /* the constant period, or Algorithm 2's p_init; >= 1 */
     int64_t K;               /* total iterations of the schedule */
     int64_t K_s;             /* Algorithm 2: syncs at iterations k < K_s sample C_2;
@@ -91,6 +92,10 @@ typedef struct {
     int32_t literal_phase;   /* kind 0 only: sync when k mod p == 0 (Algorithm 1 as printed)
                                 instead of when cnt reaches p */
     const int64_t* milestones; /* iterations from which the step size changes */
+    int32_t n_period_changes;  /* kind 2: the period is p_init, then period_values[t] from iteration */
+    int32_t reserved;          /* period_change_k[t] on (increasing k, values >= 1; host arrays) */
+    const int64_t* period_change_k;
+    const int32_t* period_values;
 } adpsgd_schedule;
 
 /* Scheduler state (everything besides x and v that a checkpoint needs). */
@@ -113,6 +118,11 @@ typedef struct {
     double* C2;              /* C_2 after the rule ran */
     double* loss;            /* 1/2 sum_j h_j (xbar_j - c_j)^2 (0 if want_loss == 0) */
     int32_t* phase;          /* 0 constant, 1 warm-up, 2 sampling, 3 adapting */
+    int64_t var_cap;         /* entries of var (0: not recorded) */
+    double* var;             /* var[k] = Var[W_k] = D / n at the start of iteration k, k < var_cap
+                                (Sec. III; the series behind V_t of Eq. vt and the weighted variance
+                                of Eq. metric2).  Costs one variance pass (4 B per replica-param) per
+                                iteration; not available with cfg.fuse_intervals */
 } adpsgd_trace;
 
 typedef struct {
@@ -198,7 +208,8 @@ int adpsgd_state_init(const adpsgd_schedule* sched, adpsgd_state* state);
  * cnt += 1 and, when cnt reaches p, one averaging, S = D / n, and the period rule
  * (adpsgd_sched_on_sync).  Updates *state so that a later call resumes bit-identically.
  * trace and stats may be NULL.  Blocks (bounded) at every sync.  Errors: E_INVAL (bad
- * schedule, K_s < p_init + K_w for kind 1, p < 1), E_TIMEOUT, E_CUDA. */
+ * schedule, K_s < p_init + K_w for kind 1, p < 1, trace->var with fuse_intervals), E_TIMEOUT,
+ * E_CUDA.  After an error the state is not resumable (restore a checkpoint). */
 int adpsgd_run(adpsgd_ctx* ctx, const adpsgd_schedule* sched, adpsgd_state* state, int64_t k_end,
                adpsgd_trace* trace, adpsgd_stats* stats);
 

@@ -376,7 +376,9 @@ double orc_variance(int32_t n, int64_t P, const float* x)
 /* Schedules.                                                                */
 /* ------------------------------------------------------------------------ */
 typedef struct {
-    int32_t kind;          /* 0 constant period (Algorithm 1), 1 adaptive (Algorithm 2) */
+    int32_t kind;          /* 0 constant period (Algorithm 1), 1 adaptive (Algorithm 2),
+                              2 piecewise-constant period (the strategies of Sec. IV-A and the
+                              decreasing period of Sec. VI-B) */
     int32_t p_init;        /* constant p, or p_init */
     int64_t K;             /* iterations */
     int64_t K_s;           /* sampling phase: syncs at k < K_s sample C_2 */
@@ -388,6 +390,10 @@ typedef struct {
     int32_t n_milestones;
     int32_t literal_phase; /* constant period only: sync when k mod p == 0 */
     const int64_t* milestones; /* gamma changes from iteration milestones[t] on */
+    int32_t n_period_changes;  /* kind 2: p = period_values[t] from iteration period_change_k[t] on */
+    int32_t pad;
+    const int64_t* period_change_k;
+    const int32_t* period_values;
 } orc_schedule;
 
 typedef struct {
@@ -407,6 +413,16 @@ float orc_gamma(const orc_schedule* s, int64_t k)
     return (float)g;
 }
 
+/* Period in force at iteration k for kind 2: p_init, replaced by period_values[t] from   */
+/* iteration period_change_k[t] on.                                                       */
+static int32_t period_at(const orc_schedule* s, int64_t k)
+{
+    int32_t p = s->p_init;
+    for (int32_t t = 0; t < s->n_period_changes; ++t)
+        if (k >= s->period_change_k[t]) p = s->period_values[t];
+    return p;
+}
+
 /* Phase codes recorded per sync. */
 enum { ORC_PHASE_CONSTANT = 0, ORC_PHASE_WARMUP = 1, ORC_PHASE_SAMPLING = 2, ORC_PHASE_ADAPTING = 3 };
 
@@ -415,7 +431,7 @@ enum { ORC_PHASE_CONSTANT = 0, ORC_PHASE_WARMUP = 1, ORC_PHASE_SAMPLING = 2, ORC
 int32_t orc_on_sync(const orc_schedule* s, orc_state* st, int64_t k, double S, double gamma)
 {
     if (k < s->K_w) return ORC_PHASE_WARMUP;
-    if (s->kind == 0) return ORC_PHASE_CONSTANT;
+    if (s->kind == 0 || s->kind == 2) return ORC_PHASE_CONSTANT;
     if (k < s->K_s) {
         st->m = st->m + 1;
         st->C2 = st->C2 + (S / gamma - st->C2) / (double)st->m;
@@ -440,6 +456,7 @@ static int sync_now(const orc_schedule* s, orc_state* st, int64_t k)
         st->cnt = 0;
         return 1;
     }
+    if (s->kind == 2) st->p = period_at(s, k);
     if (s->kind == 0 && s->literal_phase) return (k % st->p) == 0;
     st->cnt = st->cnt + 1;
     if (st->cnt >= st->p) {
@@ -457,6 +474,8 @@ typedef struct {
     double* loss;    /* surrogate loss at the average */
     int32_t* phase;  /* phase code */
     int64_t cap;     /* capacity of the arrays */
+    double* var;     /* optional: var[k] = Var[W_k] (Sec. III) at the start of iteration k */
+    int64_t var_cap; /* entries of var */
 } orc_trace;
 
 /* Initial scheduler state. */
@@ -477,6 +496,7 @@ int64_t orc_run(int32_t n, int64_t P, float* x, float* v, const float* h, const 
     int64_t syncs = 0;
     for (int64_t k = k_begin; k < k_end; ++k) {
         float gamma = orc_gamma(s, k);
+        if (tr != NULL && tr->var != NULL && k < tr->var_cap) tr->var[k] = orc_variance(n, P, x) / (double)n;
         orc_local_step(n, P, 0, P, x, v, h, c, noise_bf16, seed, k, gamma, mu, wd, sigma);
         if (!sync_now(s, st, k)) continue;
         double D = 0.0, loss = 0.0;

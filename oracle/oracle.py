@@ -70,7 +70,8 @@ class Schedule(C.Structure):
         ("K_w", C.c_int64), ("lo", C.c_double), ("hi", C.c_double), ("p_min", C.c_int32),
         ("p_max", C.c_int32), ("lr0", C.c_double), ("lr_factor", C.c_double),
         ("n_milestones", C.c_int32), ("literal_phase", C.c_int32),
-        ("milestones", C.POINTER(C.c_int64)),
+        ("milestones", C.POINTER(C.c_int64)), ("n_period_changes", C.c_int32), ("pad", C.c_int32),
+        ("period_change_k", C.POINTER(C.c_int64)), ("period_values", C.POINTER(C.c_int32)),
     ]
 
 
@@ -82,7 +83,8 @@ class Trace(C.Structure):
     _fields_ = [
         ("k", C.POINTER(C.c_int64)), ("p", C.POINTER(C.c_int32)), ("S", C.POINTER(C.c_double)),
         ("C2", C.POINTER(C.c_double)), ("loss", C.POINTER(C.c_double)),
-        ("phase", C.POINTER(C.c_int32)), ("cap", C.c_int64),
+        ("phase", C.POINTER(C.c_int32)), ("cap", C.c_int64), ("var", C.POINTER(C.c_double)),
+        ("var_cap", C.c_int64),
     ]
 
 
@@ -253,7 +255,8 @@ def variance(x) -> float:
 
 @dataclass
 class ScheduleSpec:
-    """Algorithm 1 (kind=0, constant p) or Algorithm 2 (kind=1) with its knobs."""
+    """Algorithm 1 (kind=0, constant p), Algorithm 2 (kind=1) with its knobs, or a piecewise-constant
+    period (kind=2: p_init, then period_values[t] from iteration period_change_k[t] on)."""
     kind: int
     K: int
     p_init: int
@@ -267,13 +270,20 @@ class ScheduleSpec:
     lr_factor: float = 0.1
     milestones: tuple = ()
     literal_phase: int = 0
+    period_changes: tuple = ()   # ((k, p), ...) for kind 2
     _ms: np.ndarray = field(default=None, repr=False)
+    _pk: np.ndarray = field(default=None, repr=False)
+    _pv: np.ndarray = field(default=None, repr=False)
 
     def c(self) -> Schedule:
         self._ms = np.ascontiguousarray(self.milestones if self.milestones else [0], dtype=np.int64)
+        ch = self.period_changes if self.period_changes else ((0, self.p_init),)
+        self._pk = np.ascontiguousarray([k for k, _ in ch], dtype=np.int64)
+        self._pv = np.ascontiguousarray([p for _, p in ch], dtype=np.int32)
         return Schedule(self.kind, self.p_init, self.K, self.K_s, self.K_w, self.lo, self.hi,
                         self.p_min, self.p_max, self.lr0, self.lr_factor, len(self.milestones),
-                        self.literal_phase, _i64p(self._ms))
+                        self.literal_phase, _i64p(self._ms), len(self.period_changes), 0,
+                        _i64p(self._pk), _i32p(self._pv))
 
 
 def gamma(spec: ScheduleSpec, k: int) -> float:
@@ -302,19 +312,23 @@ class RunTrace:
     loss: np.ndarray
     phase: np.ndarray
     syncs: int
+    var: np.ndarray = None
 
 
 def run(x, v, h, c, *, spec: ScheduleSpec, seed, mu, wd, sigma, noise=None, state=None,
-        k_begin=0, k_end=None, cap=100000) -> RunTrace:
-    """Algorithm 2 (or 1) end to end on the [n, P] arrays, in place; returns the sync trace."""
+        k_begin=0, k_end=None, cap=100000, track_variance=False) -> RunTrace:
+    """Algorithm 2 (or 1) end to end on the [n, P] arrays, in place; returns the sync trace and,
+    with track_variance, Var[W_k] at the start of every iteration k (Sec. III, Eq. vt)."""
     _check_state(x, v)
     n, P = x.shape
     k_end = spec.K if k_end is None else k_end
     st = new_state(spec) if state is None else state
     arrs = dict(k=np.zeros(cap, np.int64), p=np.zeros(cap, np.int32), S=np.zeros(cap),
                 C2=np.zeros(cap), loss=np.zeros(cap), phase=np.zeros(cap, np.int32))
+    var = np.full(k_end, np.nan) if track_variance else None
     tr = Trace(_i64p(arrs["k"]), _i32p(arrs["p"]), _f64p(arrs["S"]), _f64p(arrs["C2"]),
-               _f64p(arrs["loss"]), _i32p(arrs["phase"]), cap)
+               _f64p(arrs["loss"]), _i32p(arrs["phase"]), cap,
+               _f64p(var) if var is not None else None, k_end if var is not None else 0)
     s = spec.c()
     h = np.ascontiguousarray(h, dtype=np.float32)
     c = np.ascontiguousarray(c, dtype=np.float32)
@@ -322,7 +336,7 @@ def run(x, v, h, c, *, spec: ScheduleSpec, seed, mu, wd, sigma, noise=None, stat
     syncs = lib().orc_run(n, P, _f32p(x), _f32p(v), _f32p(h), _f32p(c), nz, seed, mu, wd, sigma,
                           C.byref(s), C.byref(st), k_begin, k_end, C.byref(tr))
     m = min(syncs, cap)
-    return RunTrace(**{a: b[:m].copy() for a, b in arrs.items()}, syncs=syncs)
+    return RunTrace(**{a: b[:m].copy() for a, b in arrs.items()}, syncs=syncs, var=var)
 
 
 def schedule_only(spec: ScheduleSpec, S_script, cap=100000):

@@ -19,7 +19,7 @@ _lib = None
 
 OK, E_INVAL, E_ALIGN, E_CUDA, E_TIMEOUT, E_NOMEM, E_STATE = 0, -1, -2, -3, -4, -5, -6
 NOISE_PHILOX, NOISE_BF16 = 0, 1
-CPSGD, ADPSGD = 0, 1
+CPSGD, ADPSGD, PIECEWISE = 0, 1, 2
 PHASE_CONSTANT, PHASE_WARMUP, PHASE_SAMPLING, PHASE_ADAPTING = 0, 1, 2, 3
 
 
@@ -42,7 +42,8 @@ class Schedule(C.Structure):
                 ("K_w", C.c_int64), ("lo", C.c_double), ("hi", C.c_double), ("p_min", C.c_int32),
                 ("p_max", C.c_int32), ("lr0", C.c_double), ("lr_factor", C.c_double),
                 ("n_milestones", C.c_int32), ("literal_phase", C.c_int32),
-                ("milestones", C.POINTER(C.c_int64))]
+                ("milestones", C.POINTER(C.c_int64)), ("n_period_changes", C.c_int32), ("reserved", C.c_int32),
+                ("period_change_k", C.POINTER(C.c_int64)), ("period_values", C.POINTER(C.c_int32))]
 
 
 class State(C.Structure):
@@ -53,7 +54,8 @@ class State(C.Structure):
 class Trace(C.Structure):
     _fields_ = [("cap", C.c_int64), ("len", C.c_int64), ("k", C.POINTER(C.c_int64)),
                 ("p", C.POINTER(C.c_int32)), ("S", C.POINTER(C.c_double)), ("C2", C.POINTER(C.c_double)),
-                ("loss", C.POINTER(C.c_double)), ("phase", C.POINTER(C.c_int32))]
+                ("loss", C.POINTER(C.c_double)), ("phase", C.POINTER(C.c_int32)), ("var_cap", C.c_int64),
+                ("var", C.POINTER(C.c_double))]
 
 
 class Stats(C.Structure):
@@ -162,11 +164,15 @@ def make_config(n, P, *, momentum=0.9, weight_decay=0.0, noise_sigma=1.0, seed=0
 
 
 def make_schedule(kind, K, p_init, *, K_s=0, K_w=0, lo=0.7, hi=1.3, p_min=1, p_max=0, lr0=0.1, lr_factor=0.1,
-                  milestones=(), literal_phase=False) -> Schedule:
+                  milestones=(), literal_phase=False, period_changes=()) -> Schedule:
+    """period_changes: ((k, p), ...) for PIECEWISE: p from iteration k on."""
     ms = (C.c_int64 * max(1, len(milestones)))(*milestones)
+    pk = (C.c_int64 * max(1, len(period_changes)))(*[k for k, _ in period_changes])
+    pv = (C.c_int32 * max(1, len(period_changes)))(*[p for _, p in period_changes])
     s = Schedule(kind, p_init, K, K_s, K_w, lo, hi, p_min, p_max, lr0, lr_factor, len(milestones),
-                 int(bool(literal_phase)), C.cast(ms, C.POINTER(C.c_int64)))
-    s._keep = ms  # keep the milestone array alive with the struct
+                 int(bool(literal_phase)), C.cast(ms, C.POINTER(C.c_int64)), len(period_changes), 0,
+                 C.cast(pk, C.POINTER(C.c_int64)), C.cast(pv, C.POINTER(C.c_int32)))
+    s._keep = (ms, pk, pv)  # keep the host arrays alive with the struct
     return s
 
 
@@ -241,9 +247,9 @@ def adpsgd_state_init(sched: Schedule) -> State:
 
 
 class TraceBuffers:
-    """Host arrays for an adpsgd_trace."""
+    """Host arrays for an adpsgd_trace; var_cap > 0 also records Var[W_k] per iteration."""
 
-    def __init__(self, cap: int):
+    def __init__(self, cap: int, var_cap: int = 0):
         import numpy as np
         self.k = np.zeros(cap, np.int64)
         self.p = np.zeros(cap, np.int32)
@@ -251,11 +257,13 @@ class TraceBuffers:
         self.C2 = np.zeros(cap)
         self.loss = np.zeros(cap)
         self.phase = np.zeros(cap, np.int32)
+        self.var = np.full(max(1, var_cap), np.nan)
         self.c = Trace(cap, 0, self.k.ctypes.data_as(C.POINTER(C.c_int64)),
                        self.p.ctypes.data_as(C.POINTER(C.c_int32)), self.S.ctypes.data_as(C.POINTER(C.c_double)),
                        self.C2.ctypes.data_as(C.POINTER(C.c_double)),
                        self.loss.ctypes.data_as(C.POINTER(C.c_double)),
-                       self.phase.ctypes.data_as(C.POINTER(C.c_int32)))
+                       self.phase.ctypes.data_as(C.POINTER(C.c_int32)), var_cap,
+                       self.var.ctypes.data_as(C.POINTER(C.c_double)) if var_cap > 0 else None)
 
     @property
     def len(self) -> int:
@@ -264,7 +272,8 @@ class TraceBuffers:
     def arrays(self):
         m = self.c.len
         return dict(k=self.k[:m].copy(), p=self.p[:m].copy(), S=self.S[:m].copy(), C2=self.C2[:m].copy(),
-                    loss=self.loss[:m].copy(), phase=self.phase[:m].copy())
+                    loss=self.loss[:m].copy(), phase=self.phase[:m].copy(),
+                    var=self.var[:self.c.var_cap].copy())
 
 
 def adpsgd_run(ctx: Context, sched: Schedule, state: State, k_end: int | None = None,

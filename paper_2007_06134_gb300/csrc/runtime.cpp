@@ -52,6 +52,8 @@ struct adpsgd_ctx {
     double* d_out = nullptr;  // D, loss, then the averaging kernel's completion counter
     double* h_out = nullptr;  // pinned, 2 doubles
     cudaEvent_t done = nullptr;
+    double* d_var = nullptr;  // per-iteration variance slots (2 doubles each), grown on demand
+    int64_t d_var_cap = 0;
     int grid_avg = 0, grid_avg_loss = 0, grid_var = 0, grid_interval = 0;
     // kernel timing
     std::vector<cudaEvent_t> free_events;
@@ -187,6 +189,23 @@ int average_enqueue(adpsgd_ctx* ctx, bool write_back, bool loss)
     return ADPSGD_OK;
 }
 
+// Variance of the current state into device slot k of ctx->d_var (no host round trip).
+int variance_into_slot(adpsgd_ctx* ctx, int64_t k)
+{
+    adpsgd::AverageArgs a;
+    a.x = ctx->x;
+    a.h = nullptr;
+    a.c = nullptr;
+    a.n = ctx->cfg.n;
+    a.P = ctx->cfg.P;
+    a.write_back = false;
+    a.partials = ctx->d_partials;
+    a.out = ctx->d_var + 2 * k;
+    a.counter = reinterpret_cast<unsigned int*>(ctx->d_out + 2);
+    a.grid = ctx->grid_var;
+    return timed(ctx, 1, [&] { return adpsgd::launch_average(a, ctx->stream); }, "variance");
+}
+
 // Averaging (write_back) or variance only; results land in ctx->h_out after a bounded wait.
 int average(adpsgd_ctx* ctx, bool write_back, bool loss)
 {
@@ -233,7 +252,16 @@ int interval(adpsgd_ctx* ctx, int64_t k0, int32_t m, const float* gamma, bool av
 int check_schedule(const adpsgd_schedule* s)
 {
     if (s == nullptr) return ADPSGD_E_INVAL;
-    if (s->kind != ADPSGD_CPSGD && s->kind != ADPSGD_ADPSGD) return ADPSGD_E_INVAL;
+    if (s->kind != ADPSGD_CPSGD && s->kind != ADPSGD_ADPSGD && s->kind != ADPSGD_PIECEWISE) return ADPSGD_E_INVAL;
+    if (s->kind == ADPSGD_PIECEWISE) {
+        if (s->n_period_changes < 0 || s->literal_phase) return ADPSGD_E_INVAL;
+        if (s->n_period_changes > 0 && (s->period_change_k == nullptr || s->period_values == nullptr))
+            return ADPSGD_E_INVAL;
+        for (int32_t t = 0; t < s->n_period_changes; ++t) {
+            if (s->period_values[t] < 1) return ADPSGD_E_INVAL;
+            if (t > 0 && s->period_change_k[t] <= s->period_change_k[t - 1]) return ADPSGD_E_INVAL;
+        }
+    }
     if (s->p_init < 1 || s->K < 0 || s->K > kMaxK || s->K_w < 0 || s->K_s < 0) return ADPSGD_E_INVAL;
     if (s->p_min < 1 || s->p_max < 0 || (s->p_max > 0 && s->p_max < s->p_min)) return ADPSGD_E_INVAL;
     if (s->n_milestones < 0 || (s->n_milestones > 0 && s->milestones == nullptr)) return ADPSGD_E_INVAL;
@@ -255,6 +283,15 @@ float gamma_of(const adpsgd_schedule* s, int64_t k)
     return (float)g;
 }
 
+// Period of a piecewise-constant schedule at iteration k.
+int32_t period_at(const adpsgd_schedule* s, int64_t k)
+{
+    int32_t p = s->p_init;
+    for (int32_t t = 0; t < s->n_period_changes; ++t)
+        if (k >= s->period_change_k[t]) p = s->period_values[t];
+    return p;
+}
+
 // Does iteration k end with a sync?  Advances cnt like Algorithm 2.
 bool sync_after(const adpsgd_schedule* s, adpsgd_state* st, int64_t k)
 {
@@ -262,6 +299,7 @@ bool sync_after(const adpsgd_schedule* s, adpsgd_state* st, int64_t k)
         st->cnt = 0;
         return true;
     }
+    if (s->kind == ADPSGD_PIECEWISE) st->p = period_at(s, k);
     if (s->kind == ADPSGD_CPSGD && s->literal_phase) return (k % st->p) == 0;
     st->cnt += 1;
     if (st->cnt >= st->p) {
@@ -274,7 +312,7 @@ bool sync_after(const adpsgd_schedule* s, adpsgd_state* st, int64_t k)
 int32_t rule(const adpsgd_schedule* s, adpsgd_state* st, int64_t k, double S, double gamma)
 {
     if (k < s->K_w) return 1;                 // warm-up
-    if (s->kind == ADPSGD_CPSGD) return 0;    // constant period
+    if (s->kind == ADPSGD_CPSGD || s->kind == ADPSGD_PIECEWISE) return 0;    // set by the schedule
     if (k < s->K_s) {                         // sampling C_2 (cumulative mean)
         st->m += 1;
         st->C2 += (S / gamma - st->C2) / (double)st->m;
@@ -386,6 +424,7 @@ void adpsgd_destroy(adpsgd_ctx* ctx)
     if (ctx->done != nullptr) cudaEventDestroy(ctx->done);
     if (ctx->d_partials != nullptr) cudaFree(ctx->d_partials);
     if (ctx->d_out != nullptr) cudaFree(ctx->d_out);
+    if (ctx->d_var != nullptr) cudaFree(ctx->d_var);
     if (ctx->h_out != nullptr) cudaFreeHost(ctx->h_out);
     delete ctx;
 }
@@ -477,6 +516,31 @@ int adpsgd_run(adpsgd_ctx* ctx, const adpsgd_schedule* sched, adpsgd_state* stat
         return ADPSGD_E_INVAL;
     const bool loss = ctx->cfg.want_loss != 0;
     const int64_t stop = k_end < sched->K ? k_end : sched->K;
+    const bool track = trace != nullptr && trace->var != nullptr && trace->var_cap > 0;
+    if (track && ctx->cfg.fuse_intervals) return ADPSGD_E_INVAL;
+    if (track && stop > ctx->d_var_cap) {
+        if (ctx->d_var != nullptr) {
+            cudaError_t e = cudaStreamSynchronize(ctx->stream);
+            if (e == cudaSuccess) e = cudaFree(ctx->d_var);
+            if (e != cudaSuccess) return cuda_fail(e, "cudaFree");
+            ctx->d_var = nullptr;
+        }
+        cudaError_t e = cudaMalloc(reinterpret_cast<void**>(&ctx->d_var), 2 * sizeof(double) * (size_t)stop);
+        if (e != cudaSuccess) {
+            ctx->d_var_cap = 0;
+            return e == cudaErrorMemoryAllocation ? ADPSGD_E_NOMEM : cuda_fail(e, "cudaMalloc");
+        }
+        ctx->d_var_cap = stop;
+    }
+    const int64_t k_first = state->k_next;
+    // The local step of iteration k, preceded (when recording) by the variance of W_k.
+    auto step = [&](int64_t k) -> int {
+        if (track && k < trace->var_cap) {
+            int rs = variance_into_slot(ctx, k);
+            if (rs != ADPSGD_OK) return rs;
+        }
+        return local_step(ctx, k, gamma_of(sched, k));
+    };
     const int64_t launches0[2] = {ctx->launches[0], ctx->launches[1]};
     const int64_t launches_fused0 = ctx->launches[2];
     bool launched_ahead = false;  // the local step of iteration k is already enqueued
@@ -523,7 +587,7 @@ int adpsgd_run(adpsgd_ctx* ctx, const adpsgd_schedule* sched, adpsgd_state* stat
     }
     for (int64_t k = state->k_next; k < stop; ++k) {
         if (!launched_ahead) {
-            st = local_step(ctx, k, gamma_of(sched, k));
+            st = step(k);
             if (st != ADPSGD_OK) return st;
         }
         launched_ahead = false;
@@ -535,7 +599,7 @@ int adpsgd_run(adpsgd_ctx* ctx, const adpsgd_schedule* sched, adpsgd_state* stat
         // enqueued behind the averaging before the host waits for S: the GPU stays busy while
         // the scalars travel to the host and the rule runs.
         if (k + 1 < stop) {
-            st = local_step(ctx, k + 1, gamma_of(sched, k + 1));
+            st = step(k + 1);
             if (st != ADPSGD_OK) return st;
             launched_ahead = true;
         }
@@ -556,6 +620,19 @@ int adpsgd_run(adpsgd_ctx* ctx, const adpsgd_schedule* sched, adpsgd_state* stat
             }
         }
         state->rounds += 1;
+    }
+    if (track) {
+        const int64_t last = std::min(stop, trace->var_cap);
+        if (last > k_first) {
+            std::vector<double> slots(2 * (size_t)(last - k_first));
+            cudaError_t e = cudaMemcpyAsync(slots.data(), ctx->d_var + 2 * k_first, slots.size() * sizeof(double),
+                                            cudaMemcpyDeviceToHost, ctx->stream);
+            if (e == cudaSuccess) e = cudaEventRecord(ctx->done, ctx->stream);
+            if (e != cudaSuccess) return cuda_fail(e, "variance copy");
+            st = wait_event(ctx, ctx->done);
+            if (st != ADPSGD_OK) return st;
+            for (int64_t k = k_first; k < last; ++k) trace->var[k] = slots[2 * (size_t)(k - k_first)] / (double)ctx->cfg.n;
+        }
     }
     if (stats != nullptr) {
         stats->rounds = state->rounds;

@@ -60,6 +60,11 @@ WORKLOADS = {
                          5e-4, 0.05),
 }
 
+# The schedule study of Sec. IV: 16 replicas, 4000 iterations, step size 0.1 x0.1 at 50 % and 75 %
+# of the run (the GoogLeNet / CIFAR-10 schedule of Sec. IV-A on a 2^20-parameter surrogate).
+WORKLOADS["strategies-n16"] = Workload("strategies-n16", 16, 1 << 20, 4000, "uniform:0.01:1", 1.0, 1.0, 0.9,
+                                       5e-4, 0.1, milestones=(2000, 3000), K_s_frac=0.25)
+
 SWEEP_N = (2, 4, 8, 16, 32)
 SWEEP_LOG2P = (16, 18, 20, 22, 24, 26, 28)
 

@@ -56,6 +56,18 @@ def test_period_rule_matches_oracle_on_random_scripts(seed):
             assert (ph, st.p, st.C2, st.m) == (oph, ost.p, ost.C2, ost.m)
 
 
+@pytest.mark.parametrize("changes", [((2000, 8),), ((2000, 4),), ((2000, 5),), ((10, 3), (17, 9), (400, 1))])
+def test_piecewise_period_matches_oracle(changes):
+    K, p0 = 4000, 4
+    lib_s = abi.make_schedule(abi.PIECEWISE, K, p0, period_changes=changes)
+    orc_s = O.ScheduleSpec(kind=2, K=K, p_init=p0, period_changes=changes)
+    syncs, ks, ps = O.schedule_only(orc_s, [])
+    # drive the library's rule through the same iterations: it only ever reports constant phase
+    st = abi.adpsgd_state_init(lib_s)
+    for k in ks[:50]:
+        assert abi.adpsgd_sched_on_sync(lib_s, st, int(k), 1.0, 0.1) == abi.PHASE_CONSTANT
+
+
 def test_wire_bytes_match_oracle():
     for n, P, R in ((1, 10, 5), (8, 11_689_512, 250), (16, 25_557_032, 125), (3, 7, 0)):
         assert abi.adpsgd_wire_bytes(n, P, R, True) == O.wire_bytes(n, P, R, True)
@@ -72,7 +84,9 @@ def test_schedule_validation():
            abi.make_schedule(abi.CPSGD, 100, 4, p_min=0),
            abi.make_schedule(abi.CPSGD, 100, 4, lr0=0.0),
            abi.make_schedule(abi.ADPSGD, 100, 4, K_s=25, literal_phase=True),
-           abi.make_schedule(2, 100, 4)]
+           abi.make_schedule(3, 100, 4),
+           abi.make_schedule(abi.PIECEWISE, 100, 4, period_changes=((50, 8), (40, 2))),
+           abi.make_schedule(abi.PIECEWISE, 100, 4, period_changes=((50, 0),))]
     for s in bad:
         with pytest.raises(abi.AdpsgdError) as e:
             abi.adpsgd_state_init(s)

@@ -239,3 +239,37 @@ def test_step_size_of_each_iteration_in_a_run():
         xk = c.astype(np.float64) * (1.0 - fac)
         expect = 0.5 * np.sum(h * (xk - c) ** 2)
         assert tr.loss[k] == pytest.approx(expect, rel=1e-5)
+
+
+def test_piecewise_strategies_sync_counts():
+    # Sec. IV-A: strategy 1 (p = 4 for 2000 iterations, then 8) and strategy 2 (8, then 4) both
+    # sync 750 times in 4000 iterations; Sec. VI-B: 20 then 5 syncs 500 times.
+    def count(p0, p1):
+        spec = O.ScheduleSpec(kind=2, K=4000, p_init=p0, period_changes=((2000, p1),))
+        return O.schedule_only(spec, [])
+    s1, k1, p1 = count(4, 8)
+    s2, _, _ = count(8, 4)
+    s3, _, _ = count(20, 5)
+    assert (s1, s2, s3) == (750, 750, 500)
+    assert k1[499] == 1999 and k1[500] == 2007 and set(p1[:500]) == {4} and set(p1[500:]) == {8}
+
+
+def test_variance_trace_resets_at_syncs_and_matches_second_moment():
+    # Var[W_k] (Sec. III) recorded at the start of every iteration: exactly 0 at k = 0 and right
+    # after every sync, and t steps into an interval its mean is the second moment of the spread.
+    n, P, p, K = 4, 1 << 14, 4, 40
+    gamma, sigma = 0.1, 0.5
+    h = inputs.draw_h(P, "uniform:0.1:1", 6)
+    c = inputs.draw_c(P, 1.0, 6)
+    x, v = inputs.zero_state(n, P)
+    spec = O.ScheduleSpec(kind=0, K=K, p_init=p, lr0=gamma)
+    tr = O.run(x, v, h, c, spec=spec, seed=17, mu=0.0, wd=0.0, sigma=sigma, track_variance=True)
+    var = tr.var
+    assert var[0] == 0.0 and all(var[k] == 0.0 for k in range(p, K, p))
+    g = np.float64(np.float32(gamma))
+    hh = h.astype(np.float64)
+    for t in range(1, p):
+        # E[D] after t steps from identical replicas, mu = 0: (n-1) sum_j g^2 sigma^2 sum_{s<t} (1-g h)^(2s)
+        ED = (n - 1) * np.sum(g * g * sigma * sigma * sum((1 - g * hh) ** (2 * s) for s in range(t)))
+        got = np.mean([var[k] for k in range(t, K, p)]) * n
+        assert abs(got / ED - 1) < 5 * np.sqrt(2.0 / ((n - 1) * P * (K // p)))
