@@ -57,8 +57,10 @@ def measured_peaks():
 
 KERNEL_SOURCES = {
     # kernel -> (file, first line marker, end marker) of the source it is built from
-    "local_step_kernel": [("kernels.cu", "struct StepParams", "struct AvgParams"), ("noise.cuh", "", "")],
-    "average_kernel": [("kernels.cu", "struct AvgParams", "__global__ void __launch_bounds__(kThreads) philox_fill")],
+    "local_step_kernel": [("kernels.cu", "struct StepParams", "struct AvgParams"), ("noise.cuh", "", ""),
+                          ("common.cuh", "", "")],
+    "average_kernel": [("kernels.cu", "struct AvgParams", "__global__ void __launch_bounds__(kThreads) philox_fill"),
+                       ("common.cuh", "", "")],
 }
 
 
