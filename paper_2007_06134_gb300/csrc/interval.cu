@@ -3,7 +3,8 @@
 //
 // The surrogate objective is separable per column, so each thread can keep the x and v of its
 // four columns of one replica in registers for all m steps; only the averaging couples the
-// replicas of a column, through shared memory.  Per replica-param the interval moves 16 bytes
+// replicas of a column, through shared memory, where every thread of the block takes a share of
+// the tile's 128 columns.  Per replica-param the interval moves 16 bytes
 // (x, v in and out) plus 8/n for h and c instead of 16 m + 8: the kernel is bound by the noise
 // generator's arithmetic, not by HBM.  Every element goes through exactly the operations of
 // local_step_kernel and average_kernel in the same order, so results are bit-identical to the
@@ -80,10 +81,14 @@ __global__ void __launch_bounds__(kTileGroups * kMaxReplicas) interval_kernel(co
 {
     __shared__ float4 tile[kMaxReplicas][kTileGroups];
     __shared__ float4 xbar_s[kTileGroups];
+    __shared__ float4 h_s[kTileGroups];
+    __shared__ float4 c_s[kTileGroups];
     __shared__ double shared[kMaxReplicas];
     __shared__ unsigned int ticket;
     const int g = threadIdx.x;
     const int i = threadIdx.y;
+    const int tid = threadIdx.y * blockDim.x + threadIdx.x;
+    const int nthreads = blockDim.x * blockDim.y;
     const int n = p.n;
     const float nf = (float)n;
     double accD = 0.0, accL = 0.0;
@@ -150,31 +155,27 @@ __global__ void __launch_bounds__(kTileGroups * kMaxReplicas) interval_kernel(co
         }
         if (!AVG) continue;
         tile[i][g] = make_float4(xs[0], xs[1], xs[2], xs[3]);
+        if (LOSS && i == 0) {
+            h_s[g] = make_float4(hs[0], hs[1], hs[2], hs[3]);
+            c_s[g] = make_float4(cs[0], cs[1], cs[2], cs[3]);
+        }
         __syncthreads();
-        if (i == 0 && active) {
-            float xb[4], d[4];
-#pragma unroll
-            for (int r = 0; r < 4; ++r) column_stats_tile(tile, g, r, n, nf, xb[r], d[r]);
-            float l[4] = {0.f, 0.f, 0.f, 0.f};
+        // The 128 columns of the tile are shared out over the whole block: thread t takes
+        // columns t, t + 32n, ...; column col is lane col % 4 of group col / 4, so consecutive
+        // threads read consecutive words of the tile.
+        for (int col = tid; col < 4 * kTileGroups; col += nthreads) {
+            const int cg = col >> 2, r = col & 3;
+            const int64_t j = 4 * (base + cg) + r;
+            if (base + cg >= p.Q || j >= p.P) continue;
+            float xb, d;
+            column_stats_tile(tile, cg, r, n, nf, xb, d);
+            accD += (double)d;
             if (LOSS) {
-#pragma unroll
-                for (int r = 0; r < 4; ++r) {
-                    const float t = xb[r] - cs[r];
-                    l[r] = (hs[r] * t) * t;
-                }
+                const float t = xb - reinterpret_cast<const float*>(&c_s[cg])[r];
+                const float l = (reinterpret_cast<const float*>(&h_s[cg])[r] * t) * t;
+                accL += (double)l;
             }
-            if (VEC) {
-                accD += (double)((d[0] + d[1]) + (d[2] + d[3]));
-                if (LOSS) accL += (double)((l[0] + l[1]) + (l[2] + l[3]));
-            } else {
-#pragma unroll
-                for (int r = 0; r < 4; ++r)
-                    if (r < valid) {
-                        accD += (double)d[r];
-                        if (LOSS) accL += (double)l[r];
-                    }
-            }
-            xbar_s[g] = make_float4(xb[0], xb[1], xb[2], xb[3]);
+            reinterpret_cast<float*>(xbar_s)[col] = xb;
         }
         __syncthreads();
         if (active) {
@@ -193,7 +194,6 @@ __global__ void __launch_bounds__(kTileGroups * kMaxReplicas) interval_kernel(co
     if (!AVG) return;
     const double bD = block_sum_any(accD, shared);
     const double bL = LOSS ? block_sum_any(accL, shared) : 0.0;
-    const int tid = threadIdx.y * blockDim.x + threadIdx.x;
     if (tid == 0) {
         p.partials[blockIdx.x] = bD;
         p.partials[gridDim.x + blockIdx.x] = bL;
@@ -204,7 +204,6 @@ __global__ void __launch_bounds__(kTileGroups * kMaxReplicas) interval_kernel(co
     if (ticket != gridDim.x - 1) return;
     __threadfence();
     double d = 0.0, l = 0.0;
-    const int nthreads = blockDim.x * blockDim.y;
     for (int b = tid; b < (int)gridDim.x; b += nthreads) {
         d += __ldcg(p.partials + b);
         if (LOSS) l += __ldcg(p.partials + gridDim.x + b);
