@@ -171,7 +171,7 @@ def test_last_step_index_of_the_counter():
 # ---------------------------------------------------------------------------------------------
 
 @pytest.mark.parametrize("n", [1, 2, 3, 4, 5, 8, 13, 16, 17, 32, 33, 40])
-@pytest.mark.parametrize("P", [1, 7, 4096, 4099, 100003])
+@pytest.mark.parametrize("P", [1, 7, 4, 4096, 4099, 100003, 1024 * 300 + 12, 512 * 77 + 8])
 def test_average_and_variance(n, P):
     h, c = _problem(P, 3)
     x, _ = inputs.random_state(n, P, 10 + n)
