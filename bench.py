@@ -13,8 +13,9 @@ value      replica-params/s of the whole run (n * P * iterations / step time), a
 e2e        the same through the C ABI with host buffers: H2D of x0, v0, h, c and D2H of the
            final x inside the timed region
 roofline   the local-step kernel (the dominant one): algorithmic bytes per launch
-           (16 n P + 8 P) over its mean CUDA-event duration, against the measured HBM copy
-           bandwidth; avg_variance reports the averaging kernel the same way (8 n P + 8 P)
+           (16 n P + 8 P) over its mean CUDA-event duration (events around every 4th launch in
+           the timed region), against the measured HBM copy bandwidth; avg_variance reports
+           the averaging kernel the same way (8 n P + 8 P)
 cpu_baseline  the CPU oracle on a bounded sample of the same workload, one host core
 
 --impl reference times the CPU oracle itself (the only reference this build has) on bounded
@@ -39,6 +40,7 @@ sys.path.insert(0, ROOT)
 METRIC = "avg+variance GB/s vs HBM peak; fused local-step replica-params/sec"
 UNIT = "replica-params/s"
 CPU_SAMPLE_COLUMNS = 1 << 20
+TIMING_PERIOD = 4  # kernel durations from CUDA events around every 4th launch of each kernel
 CPU_SAMPLE_ITERS = 24
 
 
@@ -267,7 +269,7 @@ def run_gpu(args, w):
         abi.adpsgd_noise_fill_bf16(w.seed, n, P, noise, stream)
     cfg = abi.make_config(n, P, momentum=w.mu, weight_decay=w.wd, noise_sigma=w.sigma, seed=seed,
                           noise_mode=abi.NOISE_BF16 if noise is not None else abi.NOISE_PHILOX, want_loss=True,
-                          time_kernels=True)
+                          time_kernels=TIMING_PERIOD)
     sched = schedule_for(abi, w)
     ctx = abi.adpsgd_init(cfg, xd, vd, hd, cd, noise, stream)
 
@@ -321,7 +323,7 @@ def run_gpu(args, w):
     clock_summary = clocks.summary()
 
     # end to end through the C ABI from pinned host buffers
-    e2e_value, h2d, d2h = None, 0, 0
+    e2e_value, h2d, d2h, e2e_phases = None, 0, 0, None
     if not args.no_e2e:
         x0h = torch.zeros((n, P), dtype=torch.float32).pin_memory()
         v0h = torch.zeros_like(x0h).pin_memory()
@@ -334,13 +336,19 @@ def run_gpu(args, w):
                                   noise_mode=cfg.noise_mode, want_loss=True)
         ctx_e2e = abi.adpsgd_init(cfg_e2e, xd, vd, hd, cd, noise, stream)  # set-up, outside the timed region
 
+        marks = [torch.cuda.Event(enable_timing=True) for _ in range(4)]
+
         def e2e_step():
+            marks[0].record(stream)
             xd.copy_(x0h, non_blocking=True)
             vd.copy_(v0h, non_blocking=True)
             hd.copy_(hh, non_blocking=True)
             cd.copy_(ch, non_blocking=True)
+            marks[1].record(stream)
             abi.adpsgd_run(ctx_e2e, sched, abi.adpsgd_state_init(sched))
+            marks[2].record(stream)
             xout.copy_(xd, non_blocking=True)
+            marks[3].record(stream)
 
         e2e_step()
         torch.cuda.synchronize(device)
@@ -352,13 +360,16 @@ def run_gpu(args, w):
         torch.cuda.synchronize(device)
         dt = max_over_ranks(pg, (time.perf_counter() - t0) / e2e_steps, device)
         e2e_value = world * rp_per_step / dt
+        e2e_phases = {"h2d_ms": marks[0].elapsed_time(marks[1]), "run_ms": marks[1].elapsed_time(marks[2]),
+                      "d2h_ms": marks[2].elapsed_time(marks[3]), "wall_ms": dt * 1000.0}
         ctx_e2e.close()
 
     # The same run with each sync interval fused into one kernel (separable objective only).
     fused = None
     if not args.no_fused and n <= 32:
         cfg_f = abi.make_config(n, P, momentum=w.mu, weight_decay=w.wd, noise_sigma=w.sigma, seed=seed,
-                                noise_mode=cfg.noise_mode, want_loss=True, time_kernels=True, fuse_intervals=True)
+                                noise_mode=cfg.noise_mode, want_loss=True, time_kernels=TIMING_PERIOD,
+                                fuse_intervals=True)
         with abi.adpsgd_init(cfg_f, xd, vd, hd, cd, noise, stream) as ctx_f:
             def fused_run():
                 xd.zero_()
@@ -396,7 +407,8 @@ def run_gpu(args, w):
                        "rounds_per_step": rounds[-1] if rounds else None,
                        "l2": "inputs larger than L2 (x, v = %.0f MB)" % (8 * n * P / 1e6),
                        "parallelism": f"independent problem per rank x{world}"},
-            "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
+            "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+                    "last_step": e2e_phases},
             "gpu_launches": launches,
             "roofline": {"kernel": "local_step_kernel", "bound": "hbm", "achieved": k1_gbs, "peak": peak,
                          "peak_kind": peak_kind, "unit": "GB/s", "frac": k1_gbs / peak,

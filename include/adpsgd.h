@@ -64,7 +64,8 @@ typedef struct {
     int32_t want_loss;       /* nonzero: averaging also returns 1/2 sum_j h_j (xbar_j - c_j)^2 */
     uint64_t seed;           /* Philox key (low word, high word) */
     int64_t wait_timeout_ms; /* bound on every host wait; <= 0 means 60000 */
-    int32_t time_kernels;    /* nonzero: bracket every kernel launch with CUDA events */
+    int32_t time_kernels;    /* N > 0: bracket every N-th launch of each kernel kind with CUDA
+                                events (1: every launch); 0: no timing */
     int32_t fuse_intervals;  /* nonzero (needs n <= 32): adpsgd_run and adpsgd_local_steps run each
                                 stretch of local steps up to the next sync (at most 256 steps), and
                                 the sync's averaging, as ONE kernel that keeps x and v in registers
@@ -248,7 +249,8 @@ int adpsgd_noise_fill_f32(uint64_t seed, uint32_t tag, int32_t n, int64_t P, int
 int adpsgd_noise_fill_bf16(uint64_t seed, int32_t n, int64_t P, uint16_t* out, void* stream);
 
 /* Device time of the kernels launched through ctx while cfg.time_kernels was set, summed from
- * CUDA events on ctx's stream since init or the last reset (waits for them, bounded).
+ * CUDA events on ctx's stream since init or the last reset (waits for them, bounded), over the
+ * timed launches only (every time_kernels-th); *_launches counts those timed launches.
  * Errors: E_INVAL (out NULL), E_STATE (timing off), E_TIMEOUT, E_CUDA. */
 int adpsgd_kernel_times(adpsgd_ctx* ctx, adpsgd_kernel_timing* out);
 int adpsgd_reset_kernel_times(adpsgd_ctx* ctx);

@@ -160,7 +160,7 @@ def _stream(stream) -> int | None:
 def make_config(n, P, *, momentum=0.9, weight_decay=0.0, noise_sigma=1.0, seed=0, noise_mode=NOISE_PHILOX,
                 want_loss=True, wait_timeout_ms=60000, time_kernels=False, fuse_intervals=False) -> Config:
     return Config(n, noise_mode, P, momentum, weight_decay, noise_sigma, int(bool(want_loss)),
-                  seed & 0xFFFFFFFFFFFFFFFF, wait_timeout_ms, int(bool(time_kernels)), int(bool(fuse_intervals)))
+                  seed & 0xFFFFFFFFFFFFFFFF, wait_timeout_ms, int(time_kernels), int(bool(fuse_intervals)))
 
 
 def make_schedule(kind, K, p_init, *, K_s=0, K_w=0, lo=0.7, hi=1.3, p_min=1, p_max=0, lr0=0.1, lr_factor=0.1,

@@ -59,53 +59,71 @@ struct StepParams {
     PhiloxKeys keys;
 };
 
-// Block b handles replica i = b mod n and blocks of four columns q = (b div n) * 256 + tid, so
-// the n blocks that read the same h, c tile run back to back (the re-reads hit L2).
+// Block b handles replica i = b mod n and the column groups (four columns each)
+// q = (b div n) * kStepGroupsPerBlock + g * kStepThreads + tid, g < kStepGroups, so the n blocks
+// that read the same h, c tile run back to back (the re-reads hit L2).  Each thread issues the
+// loads of its kStepGroups groups before any arithmetic; 128-thread blocks with two groups per
+// thread measured 5 % faster than 256 threads with one.
+constexpr int kStepThreads = 128;
+constexpr int kStepGroups = 2;
+constexpr int kStepGroupsPerBlock = kStepThreads * kStepGroups;
+
 template <bool VEC, bool BF16, bool WD>
-__global__ void __launch_bounds__(kThreads) local_step_kernel(const StepParams p)
+__global__ void __launch_bounds__(kStepThreads) local_step_kernel(const StepParams p)
 {
     const int64_t b = blockIdx.x;
     const int32_t i = (int32_t)(b % p.n);
-    const int64_t q = (b / p.n) * kThreads + threadIdx.x;
-    if (q >= p.Q) return;
+    const int64_t q0 = (b / p.n) * kStepGroupsPerBlock + threadIdx.x;
     const int64_t row = (int64_t)i * p.P;
     if (VEC) {
-        float4* __restrict__ xp = reinterpret_cast<float4*>(p.x + row) + q;
-        float4* __restrict__ vp = reinterpret_cast<float4*>(p.v + row) + q;
-        float4 xv = *xp;
-        float4 vv = *vp;
-        const float4 hv = __ldg(reinterpret_cast<const float4*>(p.h) + q);
-        const float4 cv = __ldg(reinterpret_cast<const float4*>(p.c) + q);
-        float4 z;
-        if (BF16) {
-            const uint2 nb = __ldg(reinterpret_cast<const uint2*>(p.noise + row) + q);
-            z = make_float4(bf16_bits_to_float(nb.x & 0xFFFFu), __uint_as_float(nb.x & 0xFFFF0000u),
-                            bf16_bits_to_float(nb.y & 0xFFFFu), __uint_as_float(nb.y & 0xFFFF0000u));
-        } else {
-            z = normals4(p.keys, (uint32_t)q, (uint32_t)i, p.k, 0u);
-        }
-        sgd_update<WD>(xv.x, vv.x, hv.x, cv.x, z.x, p.gamma, p.mu, p.wd, p.sigma);
-        sgd_update<WD>(xv.y, vv.y, hv.y, cv.y, z.y, p.gamma, p.mu, p.wd, p.sigma);
-        sgd_update<WD>(xv.z, vv.z, hv.z, cv.z, z.z, p.gamma, p.mu, p.wd, p.sigma);
-        sgd_update<WD>(xv.w, vv.w, hv.w, cv.w, z.w, p.gamma, p.mu, p.wd, p.sigma);
-        *xp = xv;
-        *vp = vv;
-    } else {
-        float zz[4];
-        if (!BF16) {
-            const float4 z = normals4(p.keys, (uint32_t)q, (uint32_t)i, p.k, 0u);
-            zz[0] = z.x; zz[1] = z.y; zz[2] = z.z; zz[3] = z.w;
+        float4 xv[kStepGroups], vv[kStepGroups], hv[kStepGroups], cv[kStepGroups], zb[kStepGroups];
+#pragma unroll
+        for (int g = 0; g < kStepGroups; ++g) {
+            const int64_t q = q0 + g * kStepThreads;
+            if (q < p.Q) {
+                xv[g] = reinterpret_cast<const float4*>(p.x + row)[q];
+                vv[g] = reinterpret_cast<const float4*>(p.v + row)[q];
+                hv[g] = __ldg(reinterpret_cast<const float4*>(p.h) + q);
+                cv[g] = __ldg(reinterpret_cast<const float4*>(p.c) + q);
+                if (BF16) {
+                    const uint2 nb = __ldg(reinterpret_cast<const uint2*>(p.noise + row) + q);
+                    zb[g] = make_float4(bf16_bits_to_float(nb.x & 0xFFFFu), __uint_as_float(nb.x & 0xFFFF0000u),
+                                        bf16_bits_to_float(nb.y & 0xFFFFu), __uint_as_float(nb.y & 0xFFFF0000u));
+                }
+            }
         }
 #pragma unroll
-        for (int r = 0; r < 4; ++r) {
-            const int64_t j = 4 * q + r;
-            if (j >= p.P) break;
-            float xs = p.x[row + j];
-            float vs = p.v[row + j];
-            const float z = BF16 ? bf16_bits_to_float(p.noise[row + j]) : zz[r];
-            sgd_update<WD>(xs, vs, __ldg(p.h + j), __ldg(p.c + j), z, p.gamma, p.mu, p.wd, p.sigma);
-            p.x[row + j] = xs;
-            p.v[row + j] = vs;
+        for (int g = 0; g < kStepGroups; ++g) {
+            const int64_t q = q0 + g * kStepThreads;
+            if (q >= p.Q) break;
+            const float4 z = BF16 ? zb[g] : normals4(p.keys, (uint32_t)q, (uint32_t)i, p.k, 0u);
+            sgd_update<WD>(xv[g].x, vv[g].x, hv[g].x, cv[g].x, z.x, p.gamma, p.mu, p.wd, p.sigma);
+            sgd_update<WD>(xv[g].y, vv[g].y, hv[g].y, cv[g].y, z.y, p.gamma, p.mu, p.wd, p.sigma);
+            sgd_update<WD>(xv[g].z, vv[g].z, hv[g].z, cv[g].z, z.z, p.gamma, p.mu, p.wd, p.sigma);
+            sgd_update<WD>(xv[g].w, vv[g].w, hv[g].w, cv[g].w, z.w, p.gamma, p.mu, p.wd, p.sigma);
+            reinterpret_cast<float4*>(p.x + row)[q] = xv[g];
+            reinterpret_cast<float4*>(p.v + row)[q] = vv[g];
+        }
+    } else {
+        for (int g = 0; g < kStepGroups; ++g) {
+            const int64_t q = q0 + g * kStepThreads;
+            if (q >= p.Q) break;
+            float zz[4];
+            if (!BF16) {
+                const float4 z = normals4(p.keys, (uint32_t)q, (uint32_t)i, p.k, 0u);
+                zz[0] = z.x; zz[1] = z.y; zz[2] = z.z; zz[3] = z.w;
+            }
+#pragma unroll
+            for (int r = 0; r < 4; ++r) {
+                const int64_t j = 4 * q + r;
+                if (j >= p.P) break;
+                float xs = p.x[row + j];
+                float vs = p.v[row + j];
+                const float z = BF16 ? bf16_bits_to_float(p.noise[row + j]) : zz[r];
+                sgd_update<WD>(xs, vs, __ldg(p.h + j), __ldg(p.c + j), z, p.gamma, p.mu, p.wd, p.sigma);
+                p.x[row + j] = xs;
+                p.v[row + j] = vs;
+            }
         }
     }
 }
@@ -385,7 +403,7 @@ cudaError_t launch_local_step(const LocalStepArgs& a, cudaStream_t stream)
                      (a.noise_bf16 == nullptr || (reinterpret_cast<uintptr_t>(a.noise_bf16) & 7u) == 0);
     const bool bf16 = a.noise_bf16 != nullptr;
     const bool wd = a.wd != 0.0f;
-    const int64_t blocks = (int64_t)a.n * ceil_div(p.Q, kThreads);
+    const int64_t blocks = (int64_t)a.n * ceil_div(p.Q, kStepGroupsPerBlock);
     void (*kernel)(const StepParams);
     if (vec) {
         if (bf16) kernel = wd ? local_step_kernel<true, true, true> : local_step_kernel<true, true, false>;
@@ -394,7 +412,7 @@ cudaError_t launch_local_step(const LocalStepArgs& a, cudaStream_t stream)
         if (bf16) kernel = wd ? local_step_kernel<false, true, true> : local_step_kernel<false, true, false>;
         else kernel = wd ? local_step_kernel<false, false, true> : local_step_kernel<false, false, false>;
     }
-    kernel<<<(unsigned)blocks, kThreads, 0, stream>>>(p);
+    kernel<<<(unsigned)blocks, kStepThreads, 0, stream>>>(p);
     return cudaGetLastError();
 }
 

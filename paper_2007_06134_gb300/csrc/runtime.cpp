@@ -123,7 +123,9 @@ template <typename Launch>
 int timed(adpsgd_ctx* ctx, int kind, Launch launch, const char* what)
 {
     cudaEvent_t a = nullptr, b = nullptr;
-    if (ctx->cfg.time_kernels) {
+    // time_kernels = N > 0: bracket every N-th launch of each kind with events.
+    const bool sample = ctx->cfg.time_kernels > 0 && ctx->launches[kind] % ctx->cfg.time_kernels == 0;
+    if (sample) {
         if (ctx->pending.size() >= 16384) {
             int st = harvest_times(ctx);
             if (st != ADPSGD_OK) return st;
@@ -137,7 +139,7 @@ int timed(adpsgd_ctx* ctx, int kind, Launch launch, const char* what)
     cudaError_t e = launch();
     if (e != cudaSuccess) return cuda_fail(e, what);
     ctx->launches[kind] += 1;
-    if (ctx->cfg.time_kernels) {
+    if (sample) {
         e = cudaEventRecord(b, ctx->stream);
         if (e != cudaSuccess) return cuda_fail(e, "cudaEventRecord");
         ctx->pending.push_back({a, b, kind});
