@@ -358,6 +358,8 @@ def run_gpu(args, w):
         for _ in range(e2e_steps):
             e2e_step()
         torch.cuda.synchronize(device)
+        log("e2e last step: h2d %.1f ms, run %.1f ms, d2h %.1f ms" % (
+            marks[0].elapsed_time(marks[1]), marks[1].elapsed_time(marks[2]), marks[2].elapsed_time(marks[3])))
         dt = max_over_ranks(pg, (time.perf_counter() - t0) / e2e_steps, device)
         e2e_value = world * rp_per_step / dt
         e2e_phases = {"h2d_ms": marks[0].elapsed_time(marks[1]), "run_ms": marks[1].elapsed_time(marks[2]),
