@@ -97,6 +97,11 @@ typedef struct {
     int32_t reserved;          /* period_change_k[t] on (increasing k, values >= 1; host arrays) */
     const int64_t* period_change_k;
     const int32_t* period_values;
+    int32_t lr_warmup_steps;   /* step-size warm-up of Sec. V-C (0 = none): on stair
+                                  s = min(k div lr_warmup_len, lr_warmup_steps - 1) the step size is
+                                  lr0 * (s + 1) before the milestone factors */
+    int32_t reserved2;
+    int64_t lr_warmup_len;     /* iterations per stair (the paper: one epoch), >= 1 */
 } adpsgd_schedule;
 
 /* Scheduler state (everything besides x and v that a checkpoint needs). */
@@ -222,8 +227,9 @@ int adpsgd_run(adpsgd_ctx* ctx, const adpsgd_schedule* sched, adpsgd_state* stat
 int adpsgd_sched_on_sync(const adpsgd_schedule* sched, adpsgd_state* state, int64_t k, double S,
                          double gamma, int32_t* phase);
 
-/* Step size of iteration k: (float)(lr0 * lr_factor^(number of milestones <= k)), the product
- * taken in fp64.  Errors: E_INVAL. */
+/* Step size of iteration k: (float)(lr0 * w_k * lr_factor^(number of milestones <= k)), the product
+ * taken in fp64, with the warm-up multiple w_k = min(k div lr_warmup_len + 1, lr_warmup_steps)
+ * (w_k = 1 without warm-up).  Errors: E_INVAL. */
 int adpsgd_gamma(const adpsgd_schedule* sched, int64_t k, float* gamma_out);
 
 /* Bytes a ring allreduce would move per node and in total for `rounds` syncs of P fp32

@@ -394,6 +394,9 @@ typedef struct {
     int32_t pad;
     const int64_t* period_change_k;
     const int32_t* period_values;
+    int32_t lr_warmup_steps;   /* step-size warm-up (Sec. V-C): gamma = lr0 * (s + 1) on stair s,   */
+    int32_t pad2;              /* s = min(k div lr_warmup_len, lr_warmup_steps - 1); 0: no warm-up */
+    int64_t lr_warmup_len;
 } orc_schedule;
 
 typedef struct {
@@ -403,11 +406,16 @@ typedef struct {
     int64_t m;    /* number of samples in C2 */
 } orc_state;
 
-/* Step size of iteration k: lr0 times lr_factor once per milestone <= k,  */
-/* in fp64, then rounded once to the fp32 that the update uses.            */
+/* Step size of iteration k: lr0 (times the warm-up stair multiple), times */
+/* lr_factor once per milestone <= k, in fp64, then rounded once to fp32.  */
 float orc_gamma(const orc_schedule* s, int64_t k)
 {
     double g = s->lr0;
+    if (s->lr_warmup_steps > 0) {
+        int64_t stair = k / s->lr_warmup_len;
+        if (stair > s->lr_warmup_steps - 1) stair = s->lr_warmup_steps - 1;
+        g = g * (double)(stair + 1);
+    }
     for (int32_t t = 0; t < s->n_milestones; ++t)
         if (k >= s->milestones[t]) g = g * s->lr_factor;
     return (float)g;

@@ -72,6 +72,7 @@ class Schedule(C.Structure):
         ("n_milestones", C.c_int32), ("literal_phase", C.c_int32),
         ("milestones", C.POINTER(C.c_int64)), ("n_period_changes", C.c_int32), ("pad", C.c_int32),
         ("period_change_k", C.POINTER(C.c_int64)), ("period_values", C.POINTER(C.c_int32)),
+        ("lr_warmup_steps", C.c_int32), ("pad2", C.c_int32), ("lr_warmup_len", C.c_int64),
     ]
 
 
@@ -271,6 +272,8 @@ class ScheduleSpec:
     milestones: tuple = ()
     literal_phase: int = 0
     period_changes: tuple = ()   # ((k, p), ...) for kind 2
+    lr_warmup_steps: int = 0     # step-size warm-up stairs (Sec. V-C), each lr_warmup_len iterations
+    lr_warmup_len: int = 1
     _ms: np.ndarray = field(default=None, repr=False)
     _pk: np.ndarray = field(default=None, repr=False)
     _pv: np.ndarray = field(default=None, repr=False)
@@ -283,7 +286,7 @@ class ScheduleSpec:
         return Schedule(self.kind, self.p_init, self.K, self.K_s, self.K_w, self.lo, self.hi,
                         self.p_min, self.p_max, self.lr0, self.lr_factor, len(self.milestones),
                         self.literal_phase, _i64p(self._ms), len(self.period_changes), 0,
-                        _i64p(self._pk), _i32p(self._pv))
+                        _i64p(self._pk), _i32p(self._pv), self.lr_warmup_steps, 0, self.lr_warmup_len)
 
 
 def gamma(spec: ScheduleSpec, k: int) -> float:

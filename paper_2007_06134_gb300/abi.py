@@ -43,7 +43,8 @@ class Schedule(C.Structure):
                 ("p_max", C.c_int32), ("lr0", C.c_double), ("lr_factor", C.c_double),
                 ("n_milestones", C.c_int32), ("literal_phase", C.c_int32),
                 ("milestones", C.POINTER(C.c_int64)), ("n_period_changes", C.c_int32), ("reserved", C.c_int32),
-                ("period_change_k", C.POINTER(C.c_int64)), ("period_values", C.POINTER(C.c_int32))]
+                ("period_change_k", C.POINTER(C.c_int64)), ("period_values", C.POINTER(C.c_int32)),
+                ("lr_warmup_steps", C.c_int32), ("reserved2", C.c_int32), ("lr_warmup_len", C.c_int64)]
 
 
 class State(C.Structure):
@@ -164,14 +165,17 @@ def make_config(n, P, *, momentum=0.9, weight_decay=0.0, noise_sigma=1.0, seed=0
 
 
 def make_schedule(kind, K, p_init, *, K_s=0, K_w=0, lo=0.7, hi=1.3, p_min=1, p_max=0, lr0=0.1, lr_factor=0.1,
-                  milestones=(), literal_phase=False, period_changes=()) -> Schedule:
-    """period_changes: ((k, p), ...) for PIECEWISE: p from iteration k on."""
+                  milestones=(), literal_phase=False, period_changes=(), lr_warmup_steps=0,
+                  lr_warmup_len=1) -> Schedule:
+    """period_changes: ((k, p), ...) for PIECEWISE: p from iteration k on.  lr_warmup_steps > 0: the
+    step size climbs lr0, 2 lr0, ... over that many stairs of lr_warmup_len iterations (Sec. V-C)."""
     ms = (C.c_int64 * max(1, len(milestones)))(*milestones)
     pk = (C.c_int64 * max(1, len(period_changes)))(*[k for k, _ in period_changes])
     pv = (C.c_int32 * max(1, len(period_changes)))(*[p for _, p in period_changes])
     s = Schedule(kind, p_init, K, K_s, K_w, lo, hi, p_min, p_max, lr0, lr_factor, len(milestones),
                  int(bool(literal_phase)), C.cast(ms, C.POINTER(C.c_int64)), len(period_changes), 0,
-                 C.cast(pk, C.POINTER(C.c_int64)), C.cast(pv, C.POINTER(C.c_int32)))
+                 C.cast(pk, C.POINTER(C.c_int64)), C.cast(pv, C.POINTER(C.c_int32)), lr_warmup_steps, 0,
+                 lr_warmup_len)
     s._keep = (ms, pk, pv)  # keep the host arrays alive with the struct
     return s
 

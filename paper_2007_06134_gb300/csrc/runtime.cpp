@@ -268,6 +268,7 @@ int check_schedule(const adpsgd_schedule* s)
     if (s->p_min < 1 || s->p_max < 0 || (s->p_max > 0 && s->p_max < s->p_min)) return ADPSGD_E_INVAL;
     if (s->n_milestones < 0 || (s->n_milestones > 0 && s->milestones == nullptr)) return ADPSGD_E_INVAL;
     if (!(s->lr0 > 0.0) || !(s->lr_factor > 0.0)) return ADPSGD_E_INVAL;
+    if (s->lr_warmup_steps < 0 || (s->lr_warmup_steps > 0 && s->lr_warmup_len < 1)) return ADPSGD_E_INVAL;
     if (s->kind == ADPSGD_ADPSGD) {
         if (s->literal_phase) return ADPSGD_E_INVAL;
         if (!(s->lo > 0.0) || !(s->hi >= s->lo)) return ADPSGD_E_INVAL;
@@ -280,6 +281,10 @@ int check_schedule(const adpsgd_schedule* s)
 float gamma_of(const adpsgd_schedule* s, int64_t k)
 {
     double g = s->lr0;
+    if (s->lr_warmup_steps > 0) {
+        const int64_t stair = std::min<int64_t>(k / s->lr_warmup_len, s->lr_warmup_steps - 1);
+        g = g * (double)(stair + 1);
+    }
     for (int32_t t = 0; t < s->n_milestones; ++t)
         if (k >= s->milestones[t]) g = g * s->lr_factor;
     return (float)g;

@@ -110,3 +110,14 @@ def test_init_argument_checks_before_any_cuda_call():
     assert lib.adpsgd_philox_fill(0, 0, 1, 4, 0, 8, None) == abi.E_ALIGN
     assert lib.adpsgd_philox_fill(0, 0, 1, 4, 1 << 32, 16, None) == abi.E_INVAL
     lib.adpsgd_destroy(None)
+
+
+def test_step_size_warmup_matches_oracle():
+    L = 7
+    kw = dict(lr0=0.1, lr_factor=0.1, milestones=(30 * L, 60 * L), lr_warmup_steps=8, lr_warmup_len=L)
+    lib_s = abi.make_schedule(abi.CPSGD, 90 * L, 1, **kw)
+    orc_s = O.ScheduleSpec(kind=0, K=90 * L, p_init=1, **kw)
+    for k in range(90 * L):
+        assert abi.adpsgd_gamma(lib_s, k) == O.gamma(orc_s, k)
+    with pytest.raises(abi.AdpsgdError):
+        abi.adpsgd_state_init(abi.make_schedule(abi.CPSGD, 10, 1, lr_warmup_steps=2, lr_warmup_len=0))

@@ -82,3 +82,18 @@ def test_variance_record_rejected_with_fused_intervals():
         with pytest.raises(abi.AdpsgdError) as e:
             abi.adpsgd_run(ctx, sched, abi.adpsgd_state_init(sched), trace=tr)
     assert e.value.status == abi.E_INVAL
+
+
+def test_imagenet_style_schedule_run():
+    # Sec. V-C: step-size warm-up stairs, averaging every iteration during the warm-up (K_w), then
+    # Algorithm 2; the run must match the oracle bit for bit.
+    w = inputs.WORKLOADS["quadratic-n4-P1M"]
+    n, P, L = 4, 2053, 5
+    kw = dict(lr0=0.01, lr_factor=0.1, milestones=(30 * L, 60 * L), lr_warmup_steps=8, lr_warmup_len=L)
+    K = 90 * L
+    sched = abi.make_schedule(abi.ADPSGD, K, 4, K_s=8 * L + 100, K_w=8 * L, **kw)
+    spec = O.ScheduleSpec(kind=1, K=K, p_init=4, K_s=8 * L + 100, K_w=8 * L, **kw)
+    gt, stats, gx, gv, otr, x, v = _run(w, n, P, sched, spec)
+    assert np.array_equal(gt["k"], otr.k) and np.array_equal(gt["p"], otr.p)
+    assert list(gt["k"][:8 * L]) == list(range(8 * L))
+    assert np.array_equal(gx, x) and np.array_equal(gv, v)

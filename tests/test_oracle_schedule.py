@@ -273,3 +273,14 @@ def test_variance_trace_resets_at_syncs_and_matches_second_moment():
         ED = (n - 1) * np.sum(g * g * sigma * sigma * sum((1 - g * hh) ** (2 * s) for s in range(t)))
         got = np.mean([var[k] for k in range(t, K, p)]) * n
         assert abs(got / ED - 1) < 5 * np.sqrt(2.0 / ((n - 1) * P * (K // p)))
+
+
+def test_imagenet_step_size_schedule():
+    # Sec. V-C: warm-up from 0.1, +0.1 per epoch for 8 epochs (0.8), x0.1 at epochs 30 and 60.
+    L = 10  # iterations per epoch
+    spec = O.ScheduleSpec(kind=0, K=90 * L, p_init=1, lr0=0.1, lr_factor=0.1, milestones=(30 * L, 60 * L),
+                          lr_warmup_steps=8, lr_warmup_len=L)
+    expect = {0: 0.1, L - 1: 0.1, L: 0.2, 3 * L + 5: 0.4, 7 * L: 0.8, 8 * L: 0.8, 29 * L + 9: 0.8,
+              30 * L: 0.08, 59 * L: 0.08, 60 * L: 0.008, 89 * L: 0.008}
+    for k, g in expect.items():
+        assert O.gamma(spec, k) == np.float32(g), (k, O.gamma(spec, k), g)
