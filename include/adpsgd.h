@@ -26,6 +26,8 @@
  *     instead of blocking forever.
  *   - Device pointers must be 16-byte aligned (ADPSGD_E_ALIGN otherwise);
  *     P need not be a multiple of 4 (a scalar kernel variant handles that).
+ *   - A context is not thread-safe: use each one from one host thread at a time.  Separate
+ *     contexts on separate streams are independent.
  */
 #ifndef ADPSGD_H
 #define ADPSGD_H

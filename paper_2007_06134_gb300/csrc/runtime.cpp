@@ -49,8 +49,8 @@ struct adpsgd_ctx {
     int sms = 0;
     adpsgd::PhiloxKeys keys{};
     double* d_partials = nullptr;
-    double* d_out = nullptr;  // D, loss, then the averaging kernel's completion counter
-    double* h_out = nullptr;  // pinned, 2 doubles
+    double* d_out = nullptr;  // D, loss, then the averaging kernel's completion counter (4 slots)
+    double* h_out = nullptr;  // pinned copy of D and loss
     cudaEvent_t done = nullptr;
     double* d_var = nullptr;  // per-iteration variance slots (2 doubles each), grown on demand
     int64_t d_var_cap = 0;
@@ -131,17 +131,35 @@ int timed(adpsgd_ctx* ctx, int kind, Launch launch, const char* what)
             if (st != ADPSGD_OK) return st;
         }
         int st = take_event(ctx, &a);
-        if (st == ADPSGD_OK) st = take_event(ctx, &b);
         if (st != ADPSGD_OK) return st;
+        st = take_event(ctx, &b);
+        if (st != ADPSGD_OK) {
+            ctx->free_events.push_back(a);
+            return st;
+        }
         cudaError_t e = cudaEventRecord(a, ctx->stream);
-        if (e != cudaSuccess) return cuda_fail(e, "cudaEventRecord");
+        if (e != cudaSuccess) {
+            ctx->free_events.push_back(a);
+            ctx->free_events.push_back(b);
+            return cuda_fail(e, "cudaEventRecord");
+        }
     }
     cudaError_t e = launch();
-    if (e != cudaSuccess) return cuda_fail(e, what);
+    if (e != cudaSuccess) {
+        if (sample) {
+            ctx->free_events.push_back(a);
+            ctx->free_events.push_back(b);
+        }
+        return cuda_fail(e, what);
+    }
     ctx->launches[kind] += 1;
     if (sample) {
         e = cudaEventRecord(b, ctx->stream);
-        if (e != cudaSuccess) return cuda_fail(e, "cudaEventRecord");
+        if (e != cudaSuccess) {
+            ctx->free_events.push_back(a);
+            ctx->free_events.push_back(b);
+            return cuda_fail(e, "cudaEventRecord");
+        }
         ctx->pending.push_back({a, b, kind});
     }
     return ADPSGD_OK;
