@@ -97,3 +97,13 @@ def test_imagenet_style_schedule_run():
     assert np.array_equal(gt["k"], otr.k) and np.array_equal(gt["p"], otr.p)
     assert list(gt["k"][:8 * L]) == list(range(8 * L))
     assert np.array_equal(gx, x) and np.array_equal(gv, v)
+
+
+@pytest.mark.parametrize("fused", [False, True])
+def test_piecewise_change_inside_an_interval(fused):
+    w = inputs.WORKLOADS["quadratic-n4-P1M"]
+    sched = abi.make_schedule(abi.PIECEWISE, 12, 4, lr0=w.lr0, period_changes=((6, 2),))
+    spec = O.ScheduleSpec(kind=2, K=12, p_init=4, lr0=w.lr0, period_changes=((6, 2),))
+    gt, stats, gx, gv, otr, x, v = _run(w, 3, 515, sched, spec, fused=fused)
+    assert list(gt["k"]) == [3, 6, 8, 10] == list(otr.k)
+    assert np.array_equal(gx, x) and np.array_equal(gv, v)

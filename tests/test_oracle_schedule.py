@@ -284,3 +284,20 @@ def test_imagenet_step_size_schedule():
               30 * L: 0.08, 59 * L: 0.08, 60 * L: 0.008, 89 * L: 0.008}
     for k, g in expect.items():
         assert O.gamma(spec, k) == np.float32(g), (k, O.gamma(spec, k), g)
+
+
+def test_piecewise_change_inside_an_interval():
+    # p = 4 until iteration 5, p = 2 from iteration 6 on: iterations 4, 5, 6 count 1, 2, 3, and at
+    # k = 6 the period in force is already 2, so the sync falls at 6; then every 2 iterations.
+    spec = O.ScheduleSpec(kind=2, K=12, p_init=4, period_changes=((6, 2),))
+    syncs, ks, ps = O.schedule_only(spec, [])
+    assert list(ks) == [3, 6, 8, 10] and list(ps) == [4, 2, 2, 2]
+
+
+def test_piecewise_ignores_the_variance():
+    # A set period is never adapted, whatever S the syncs report.
+    spec = O.ScheduleSpec(kind=2, K=400, p_init=4, K_s=0, period_changes=((200, 8),))
+    _, ks, ps = O.schedule_only(spec, np.full(200, 5.0))
+    assert set(ps[:50]) == {4} and set(ps[50:]) == {8}
+    st = O.new_state(spec)
+    assert O.on_sync(spec, st, 10, 5.0, 0.1) == O.PHASE_CONSTANT and st.p == 4
