@@ -394,6 +394,38 @@ def run_gpu(args, w):
                  "note": "each sync interval (local steps + averaging) as one kernel; valid for the "
                          "separable surrogate objective only, not for a real model"}
 
+    # The paper's comparison for this workload: ADPSGD against CPSGD at the same number of averaging
+    # rounds (p = round(K / R)), and full-communication SGD (one allreduce per iteration), as rounds,
+    # equivalent period, final loss and the bytes a ring allreduce would move per node.
+    comparison = None
+    if not args.no_compare:
+        tr_a = abi.TraceBuffers(w.K + 1)
+        xd.zero_()
+        vd.zero_()
+        sa = abi.adpsgd_run(ctx, sched, abi.adpsgd_state_init(sched), trace=tr_a)
+        ta = tr_a.arrays()
+        p_eq = max(1, round(w.K / max(1, sa.rounds)))
+        rows = {"adpsgd": (sched, sa, ta)}
+        for label, p_c in (("cpsgd_equal_budget", p_eq), ("cpsgd_p%d" % w.cpsgd_p, w.cpsgd_p)):
+            if label in rows or (label != "cpsgd_equal_budget" and p_c == p_eq):
+                continue
+            sc = abi.make_schedule(abi.CPSGD, w.K, p_c, lr0=w.lr0, lr_factor=w.lr_factor, milestones=w.milestones)
+            tr_c = abi.TraceBuffers(w.K + 1)
+            xd.zero_()
+            vd.zero_()
+            st_c = abi.adpsgd_run(ctx, sc, abi.adpsgd_state_init(sc), trace=tr_c)
+            rows[label] = (sc, st_c, tr_c.arrays())
+        comparison = {}
+        for label, (sc, stt, tt) in rows.items():
+            comparison[label] = {"p": int(sc.p_init), "rounds": int(stt.rounds), "equiv_period": stt.equiv_period,
+                                 "k_last_sync": int(tt["k"][-1]) if len(tt["k"]) else None,
+                                 "loss_at_last_sync": float(tt["loss"][-1]) if len(tt["loss"]) else None,
+                                 "S_at_last_sync": float(tt["S"][-1]) if len(tt["S"]) else None,
+                                 "wire_bytes_per_node": stt.wire_bytes_per_node,
+                                 "wire_bytes_total": stt.wire_bytes_total}
+        full_pn, full_tot = abi.adpsgd_wire_bytes(n, P, w.K, False)
+        comparison["fullsgd"] = {"p": 1, "rounds": w.K, "wire_bytes_per_node": full_pn, "wire_bytes_total": full_tot}
+
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu:
         r, dt, sample = oracle_sample(w)
@@ -422,6 +454,7 @@ def run_gpu(args, w):
                              "traffic": recorded_traffic("average_kernel", w.name)},
             "local_step_rp_per_s": n * P / (k1_ms / 1000.0),
             "fused_intervals": fused,
+            "comparison": comparison,
             "clocks": clock_summary,
             "cpu_baseline": cpu,
         }
@@ -537,6 +570,7 @@ def main():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu", action="store_true")
     ap.add_argument("--no-fused", action="store_true", help="skip the fused-interval measurement")
+    ap.add_argument("--no-compare", action="store_true", help="skip the ADPSGD / CPSGD / FULLSGD comparison runs")
     ap.add_argument("--sweep", action="store_true", help="averaging-kernel sweep over n x P instead")
     ap.add_argument("--sweep-max-bytes", type=float, default=70e9)
     ap.add_argument("--variance-traces", action="store_true",
