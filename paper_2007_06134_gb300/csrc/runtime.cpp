@@ -13,12 +13,20 @@
 #include <thread>
 #include <vector>
 
+#include <nvtx3/nvToolsExt.h>
+
 #include "../../include/adpsgd.h"
 #include "launch.h"
 
 namespace {
 
 thread_local std::string g_last_error;
+
+// NVTX range for profiler timelines (header-only NVTX 3; a no-op without a tool attached).
+struct NvtxRange {
+    explicit NvtxRange(const char* name) { nvtxRangePushA(name); }
+    ~NvtxRange() { nvtxRangePop(); }
+};
 
 int cuda_fail(cudaError_t e, const char* where)
 {
@@ -457,6 +465,7 @@ void adpsgd_destroy(adpsgd_ctx* ctx)
 int adpsgd_local_steps(adpsgd_ctx* ctx, int64_t k0, int32_t m, const float* lr)
 {
     if (ctx == nullptr || m < 0 || k0 < 0 || k0 + m > kMaxK || (m > 0 && lr == nullptr)) return ADPSGD_E_INVAL;
+    NvtxRange range("adpsgd_local_steps");
     if (ctx->cfg.fuse_intervals) {
         for (int32_t t = 0; t < m; t += adpsgd::kMaxFusedSteps) {
             const int32_t chunk = std::min<int32_t>(adpsgd::kMaxFusedSteps, m - t);
@@ -475,6 +484,7 @@ int adpsgd_local_steps(adpsgd_ctx* ctx, int64_t k0, int32_t m, const float* lr)
 int adpsgd_average_and_variance(adpsgd_ctx* ctx, double* D_out, double* loss_out)
 {
     if (ctx == nullptr || D_out == nullptr) return ADPSGD_E_INVAL;
+    NvtxRange range("adpsgd_average_and_variance");
     if (loss_out != nullptr && !ctx->cfg.want_loss) return ADPSGD_E_STATE;
     int st = average(ctx, true, loss_out != nullptr);
     if (st != ADPSGD_OK) return st;
@@ -532,6 +542,7 @@ int adpsgd_run(adpsgd_ctx* ctx, const adpsgd_schedule* sched, adpsgd_state* stat
                adpsgd_trace* trace, adpsgd_stats* stats)
 {
     if (ctx == nullptr || state == nullptr) return ADPSGD_E_INVAL;
+    NvtxRange range("adpsgd_run");
     int st = check_schedule(sched);
     if (st != ADPSGD_OK) return st;
     if (state->p < 1 || state->k_next < 0 || state->cnt < 0) return ADPSGD_E_INVAL;
@@ -590,7 +601,10 @@ int adpsgd_run(adpsgd_ctx* ctx, const adpsgd_schedule* sched, adpsgd_state* stat
             if (st != ADPSGD_OK) return st;
             state->k_next = k + m;
             if (sync) {
-                st = wait_event(ctx, ctx->done);
+                {
+                    NvtxRange wait_range("adpsgd_sync_wait");
+                    st = wait_event(ctx, ctx->done);
+                }
                 if (st != ADPSGD_OK) return st;
                 const int64_t ks = k + m - 1;
                 const double S = ctx->h_out[0] / (double)ctx->cfg.n;
@@ -628,7 +642,10 @@ int adpsgd_run(adpsgd_ctx* ctx, const adpsgd_schedule* sched, adpsgd_state* stat
             if (st != ADPSGD_OK) return st;
             launched_ahead = true;
         }
-        st = wait_event(ctx, ctx->done);
+        {
+            NvtxRange wait_range("adpsgd_sync_wait");
+            st = wait_event(ctx, ctx->done);
+        }
         if (st != ADPSGD_OK) return st;
         const double S = ctx->h_out[0] / (double)ctx->cfg.n;
         const int32_t phase = rule(sched, state, k, S, (double)gamma_of(sched, k));
