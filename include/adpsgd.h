@@ -242,13 +242,13 @@ int adpsgd_wire_bytes(int32_t n, int64_t P, int64_t rounds, int32_t with_scalar,
 
 /* Raw Philox4x32-10 words of the noise stream: out[(i * nq + q) * 4 + r] = word r of
  * Philox(counter (q, i, k, tag), key (seed lo, seed hi)), i < n, q < nq.  out: device
- * uint32 [n, nq, 4].  Enqueued only.  Errors: E_INVAL, E_ALIGN, E_CUDA. */
+ * uint32 [n, nq, 4].  Enqueued only.  Errors: E_INVAL (n * nq > 2^38, k >= 2^32), E_ALIGN, E_CUDA. */
 int adpsgd_philox_fill(uint64_t seed, uint32_t tag, int32_t n, int64_t nq, int64_t k,
                        uint32_t* out, void* stream);
 
 /* The fp32 normals the local step uses: out[i * P + j] = z[i, j] of stream `tag` at step k
  * (Box-Muller of words (0,1) -> elements 4q, 4q+1 and (2,3) -> 4q+2, 4q+3).  out: device fp32
- * [n, P].  Enqueued only.  Errors: E_INVAL, E_ALIGN, E_CUDA. */
+ * [n, P].  Enqueued only.  Errors: E_INVAL (n * P > 2^40, P > 2^34), E_ALIGN, E_CUDA. */
 int adpsgd_noise_fill_f32(uint64_t seed, uint32_t tag, int32_t n, int64_t P, int64_t k,
                           float* out, void* stream);
 

@@ -749,6 +749,7 @@ int adpsgd_average_and_variance_static(float* x, const float* h, const float* c,
 int adpsgd_philox_fill(uint64_t seed, uint32_t tag, int32_t n, int64_t nq, int64_t k, uint32_t* out, void* stream)
 {
     if (out == nullptr || n < 0 || nq < 0 || nq > kMaxK || k < 0 || k >= kMaxK) return ADPSGD_E_INVAL;
+    if ((int64_t)n * nq > (int64_t(1) << 38)) return ADPSGD_E_INVAL;  // keeps the grid below 2^31 blocks
     if (!aligned16(out)) return ADPSGD_E_ALIGN;
     cudaError_t e = adpsgd::launch_philox_fill(seed, tag, n, nq, (uint32_t)k, out, static_cast<cudaStream_t>(stream));
     return e == cudaSuccess ? ADPSGD_OK : cuda_fail(e, "philox fill");
@@ -757,6 +758,7 @@ int adpsgd_philox_fill(uint64_t seed, uint32_t tag, int32_t n, int64_t nq, int64
 int adpsgd_noise_fill_f32(uint64_t seed, uint32_t tag, int32_t n, int64_t P, int64_t k, float* out, void* stream)
 {
     if (out == nullptr || n < 0 || P < 0 || P > (int64_t(1) << 34) || k < 0 || k >= kMaxK) return ADPSGD_E_INVAL;
+    if ((int64_t)n * P > (int64_t(1) << 40)) return ADPSGD_E_INVAL;
     if (!aligned16(out)) return ADPSGD_E_ALIGN;
     cudaError_t e = adpsgd::launch_noise_f32(seed, tag, n, P, (uint32_t)k, out, static_cast<cudaStream_t>(stream));
     return e == cudaSuccess ? ADPSGD_OK : cuda_fail(e, "noise fill");
@@ -765,6 +767,7 @@ int adpsgd_noise_fill_f32(uint64_t seed, uint32_t tag, int32_t n, int64_t P, int
 int adpsgd_noise_fill_bf16(uint64_t seed, int32_t n, int64_t P, uint16_t* out, void* stream)
 {
     if (out == nullptr || n < 0 || P < 0 || P > (int64_t(1) << 34)) return ADPSGD_E_INVAL;
+    if ((int64_t)n * P > (int64_t(1) << 40)) return ADPSGD_E_INVAL;
     if (!aligned16(out)) return ADPSGD_E_ALIGN;
     cudaError_t e = adpsgd::launch_noise_bf16(seed, n, P, out, static_cast<cudaStream_t>(stream));
     return e == cudaSuccess ? ADPSGD_OK : cuda_fail(e, "bf16 noise fill");

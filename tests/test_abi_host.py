@@ -109,6 +109,12 @@ def test_init_argument_checks_before_any_cuda_call():
     assert lib.adpsgd_philox_fill(0, 0, 1, 4, 0, None, None) == abi.E_INVAL
     assert lib.adpsgd_philox_fill(0, 0, 1, 4, 0, 8, None) == abi.E_ALIGN
     assert lib.adpsgd_philox_fill(0, 0, 1, 4, 1 << 32, 16, None) == abi.E_INVAL
+    assert lib.adpsgd_philox_fill(0, 0, 1 << 20, 1 << 30, 0, 16, None) == abi.E_INVAL
+    assert lib.adpsgd_noise_fill_f32(0, 0, 1 << 10, 1 << 34, 0, 16, None) == abi.E_INVAL
+    assert lib.adpsgd_noise_fill_bf16(0, 1 << 10, 1 << 34, 16, None) == abi.E_INVAL
+    assert lib.adpsgd_noise_fill_bf16(0, 1, (1 << 34) + 1, 16, None) == abi.E_INVAL
+    big = abi.make_config(1 << 10, 1 << 34)
+    assert lib.adpsgd_init(C.byref(big), 16, 32, 48, 64, None, None, C.byref(out)) == abi.E_INVAL
     lib.adpsgd_destroy(None)
 
 
