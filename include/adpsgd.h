@@ -176,6 +176,11 @@ int adpsgd_local_steps(adpsgd_ctx* ctx, int64_t k0, int32_t m, const float* lr);
  * all n replicas, and *D_out = sum_j sum_i (x_ij - xbar_j)^2 over the pre-average values
  * (n * Var[W]), accumulated in fp64.  If loss_out != NULL (needs cfg.want_loss),
  * *loss_out = 1/2 sum_j h_j (xbar_j - c_j)^2.  Blocks (bounded) until the scalars arrive.
+ * Accuracy (every averaging entry point, and the syncs of adpsgd_run): xbar as written above,
+ * bit for bit.  D and the loss are within 1e-4 relative of the fp64 definitions, over the
+ * whole fp32 range, for h_j >= 0.  Squares are taken in fp32 where their column sums lie in
+ * [2^-100, 2^100].  Elsewhere the columns are redone in fp64: subnormal or huge deviations,
+ * inf, NaN.  A NaN or inf in x gives a NaN or inf D, as the definition does.
  * Errors: E_INVAL (D_out NULL), E_STATE (loss requested without want_loss), E_TIMEOUT, E_CUDA. */
 int adpsgd_average_and_variance(adpsgd_ctx* ctx, double* D_out, double* loss_out);
 
@@ -186,7 +191,7 @@ int adpsgd_average_and_variance(adpsgd_ctx* ctx, double* D_out, double* loss_out
  * this is an interface variant, not part of the method.
  *
  * It needs no context and allocates nothing.  Its scratch is a fixed array inside the library,
- * 2 * 2048 + 2 doubles (32.8 KB), which every GPU that loads the library holds until the process
+ * 2 * 2048 + 4 doubles (32.8 KB), which every GPU that loads the library holds until the process
  * exits.  The per-block partial sums for up to 2048 blocks live there.  A shape whose averaging
  * grid would need more blocks is rejected with ADPSGD_E_INVAL; on GB300 the grid is at most
  * 1216 blocks.
@@ -197,8 +202,8 @@ int adpsgd_average_and_variance(adpsgd_ctx* ctx, double* D_out, double* loss_out
  *
  * The first call on each device looks up the scratch array's device address
  * (cudaGetSymbolAddress).  Make that first call before any stream capture.  Every call uses the
- * same array, which keeps the last call's contents.  Each call writes every slot it later reads,
- * so nothing needs clearing between calls.  Calls that overlap on the GPU (several host threads,
+ * same array, which keeps the last call's contents.  Each call clears the completion counter in
+ * it on the stream before the launch, and writes every other slot before reading it.  Calls that overlap on the GPU (several host threads,
  * or streams that run concurrently) race on the array and must be serialised by the caller.
  * Errors: E_INVAL, E_ALIGN, E_TIMEOUT, E_CUDA. */
 int adpsgd_average_and_variance_static(float* x, const float* h, const float* c, int32_t n, int64_t P,

@@ -47,15 +47,21 @@ __device__ __forceinline__ double block_sum(double v, double* shared)
 }
 
 // Per-column statistics of one column held as values r_0 .. r_{n-1}:
-// xbar = r_0 + (sum_{i>=1} (r_i - r_0)) / n   and   d = sum_i (r_i - xbar)^2  (fp32).
+// xbar = r_0 + (sum_{i>=1} (r_i - r_0)) / n   and   d = sum_i (r_i - xbar)^2  (fp32), and
+// z = sum_{i>=1} |r_i - r_0|, which is zero exactly when all n values are equal.
 template <int NMAX>
-__device__ __forceinline__ void column_stats(const float* r, int n, float nf, float& xbar, float& d)
+__device__ __forceinline__ void column_stats(const float* r, int n, float nf, float& xbar, float& d, float& z)
 {
     const float base = r[0];
-    float acc = 0.0f;
+    float acc = 0.0f, spread = 0.0f;
 #pragma unroll
     for (int i = 1; i < NMAX; ++i)
-        if (i < n) acc = acc + (r[i] - base);
+        if (i < n) {
+            const float diff = r[i] - base;
+            acc = acc + diff;
+            spread = spread + fabsf(diff);
+        }
+    z = spread;
     xbar = base + __fdiv_rn(acc, nf);
     float s = 0.0f;
 #pragma unroll
@@ -65,6 +71,75 @@ __device__ __forceinline__ void column_stats(const float* r, int n, float nf, fl
             s = s + dev * dev;
         }
     d = s;
+}
+
+// A column's fp32 sum of squared deviations (or its loss term h t^2) is within about n 2^-24 of
+// its exact value while it lies in [2^-100, 2^100]: no square in it has overflowed, and a square
+// that underflowed (below 2^-126) is negligible beside the sum.  Outside that range -- deviations
+// below about 2^-50 or above 2^50, an infinity, a NaN -- the column is recomputed in fp64 from the
+// fp32 values, which holds for any fp32 input, unless the fp32 result is an exact zero.  The
+// workloads stay in the range; the fp64 path (slow on this part) only runs for such columns.
+__device__ __forceinline__ bool sum_sq_in_range(float s) { return s >= 0x1p-100f && s <= 0x1p100f; }
+
+// A loss term l = (h t) t that is exactly zero because t = 0, or h = 0 with t finite.
+__device__ __forceinline__ bool loss_term_exact_zero(float l, float h, float t)
+{
+    return l == 0.0f && (t == 0.0f || (h == 0.0f && fabsf(t) <= 0x1.fffffep127f));
+}
+
+// A loss term whose fp32 value can be used: in range (|l|, so that a negative curvature h takes
+// no fp64 path either) or an exact zero.
+__device__ __forceinline__ bool loss_term_usable(float l, float h, float t)
+{
+    return sum_sq_in_range(fabsf(l)) || loss_term_exact_zero(l, h, t);
+}
+
+// Whether every value get(i), i < n, equals xbar: with an fp32 sum of zero this makes the
+// column's squared deviations exactly zero.
+template <int NMAX, class Get>
+__device__ __forceinline__ bool all_equal(const Get& get, int n, float xbar)
+{
+    const int m = NMAX > 0 ? NMAX : n;  // NMAX = 0: any n
+    bool eq = true;
+#pragma unroll
+    for (int i = 0; i < m; ++i)
+        if (i < n) eq = eq && get(i) == xbar;
+    return eq;
+}
+
+// sum_i (get(i) - xbar)^2 in fp64.
+template <int NMAX, class Get>
+__device__ __forceinline__ double sq_dev_f64(const Get& get, int n, float xbar)
+{
+    const int m = NMAX > 0 ? NMAX : n;
+    const double xb = (double)xbar;
+    double s = 0.0;
+#pragma unroll
+    for (int i = 0; i < m; ++i)
+        if (i < n) {
+            const double dev = (double)get(i) - xb;
+            s = s + dev * dev;
+        }
+    return s;
+}
+
+// A column's squared deviations from its fp32 sum d: d itself when usable, else fp64.
+template <int NMAX, class Get>
+__device__ __forceinline__ double checked_sq_dev(const Get& get, int n, float xbar, float d)
+{
+    if (sum_sq_in_range(d)) return (double)d;
+    if (d == 0.0f && all_equal<NMAX>(get, n, xbar)) return 0.0;
+    return sq_dev_f64<NMAX>(get, n, xbar);
+}
+
+// A column's loss term h (xbar - c)^2 (before the factor 1/2): the fp32 value when usable, else fp64.
+__device__ __forceinline__ double checked_loss_term(float h, float xbar, float c)
+{
+    const float t = xbar - c;
+    const float l = (h * t) * t;
+    if (loss_term_usable(l, h, t)) return (double)l;
+    const double td = (double)xbar - (double)c;
+    return ((double)h * td) * td;
 }
 
 }  // namespace adpsgd

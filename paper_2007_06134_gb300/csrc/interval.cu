@@ -169,12 +169,10 @@ __global__ void __launch_bounds__(kTileGroups * kMaxReplicas) interval_kernel(co
             if (base + cg >= p.Q || j >= p.P) continue;
             float xb, d;
             column_stats_tile(tile, cg, r, n, nf, xb, d);
-            accD += (double)d;
-            if (LOSS) {
-                const float t = xb - reinterpret_cast<const float*>(&c_s[cg])[r];
-                const float l = (reinterpret_cast<const float*>(&h_s[cg])[r] * t) * t;
-                accL += (double)l;
-            }
+            accD += checked_sq_dev<0>([&](int t) { return reinterpret_cast<const float*>(&tile[t][cg])[r]; }, n, xb, d);
+            if (LOSS)
+                accL += checked_loss_term(reinterpret_cast<const float*>(&h_s[cg])[r], xb,
+                                          reinterpret_cast<const float*>(&c_s[cg])[r]);
             reinterpret_cast<float*>(xbar_s)[col] = xb;
         }
         __syncthreads();

@@ -145,11 +145,16 @@ struct AvgParams {
 
 // Columns with more than 32 replicas: the same arithmetic, re-reading x (L1/L2) per pass.
 __device__ __forceinline__ void column_stats_global(const float* x, int64_t P, int64_t j, int n, float nf,
-                                                    float& xbar, float& d)
+                                                    float& xbar, float& d, float& z)
 {
     const float base = x[j];
-    float acc = 0.0f;
-    for (int i = 1; i < n; ++i) acc = acc + (x[(int64_t)i * P + j] - base);
+    float acc = 0.0f, spread = 0.0f;
+    for (int i = 1; i < n; ++i) {
+        const float diff = x[(int64_t)i * P + j] - base;
+        acc = acc + diff;
+        spread = spread + fabsf(diff);
+    }
+    z = spread;
     xbar = base + __fdiv_rn(acc, nf);
     float s = 0.0f;
     for (int i = 0; i < n; ++i) {
@@ -177,44 +182,113 @@ template <> struct ColumnGroup<false> {
     static __device__ __forceinline__ float make(const float* f) { return f[0]; }
 };
 
-// Statistics, loss and write-back of column group q whose replica values are vals[0..n).
+// A column group's fp32 sums can be added as they are when each lies in the accurate range of
+// sum_sq_in_range or is an exact zero: the squared deviations d when every column's values are all
+// equal (z = 0), the loss terms when each is zero because t = 0, or h = 0 with t finite.  The
+// first pass (finish_group) adds a group's d and writes it back when d is usable, and adds its
+// loss when both are usable.  The second pass (redo_group) recomputes the same decisions and adds
+// the rest.
+template <int W>
+__device__ __forceinline__ float group_sum(const float* a)
+{
+    return W == 4 ? (a[0] + a[W > 1 ? 1 : 0]) + (a[W > 2 ? 2 : 0] + a[W > 3 ? 3 : 0]) : a[0];
+}
+
+template <int W>
+__device__ __forceinline__ bool dev_usable(const float* d, const float* z)
+{
+    const float dsum = group_sum<W>(d);
+    return sum_sq_in_range(dsum) || (dsum == 0.0f && group_sum<W>(z) == 0.0f);
+}
+
+template <int W>
+__device__ __forceinline__ bool loss_usable(const float* l, const float* hs, const float* ts)
+{
+    if (sum_sq_in_range(fabsf(group_sum<W>(l)))) return true;
+    bool zero = true;
+#pragma unroll
+    for (int r = 0; r < W; ++r) zero = zero && loss_term_exact_zero(l[r], hs[r], ts[r]);
+    return zero;
+}
+
+// Statistics, loss and write-back of column group q whose replica values are vals[0..n), all in
+// fp32 and without branches.  Returns false when part of the group is left to redo_group.
 template <int R, bool VEC, bool LOSS, bool WRITE>
-__device__ __forceinline__ void finish_group(const AvgParams& p, int64_t q, const typename ColumnGroup<VEC>::T* vals,
+__device__ __forceinline__ bool finish_group(const AvgParams& p, int64_t q, const typename ColumnGroup<VEC>::T* vals,
                                              float nf, double& accD, double& accL)
 {
     using G = ColumnGroup<VEC>;
     constexpr int W = G::W;
-    float xbar[W], d[W];
+    float xbar[W], d[W], z[W];
 #pragma unroll
     for (int r = 0; r < W; ++r) {
         float col[R];
 #pragma unroll
         for (int i = 0; i < R; ++i) col[i] = (i < p.n) ? G::lane(vals[i], r) : 0.0f;
-        column_stats<R>(col, p.n, nf, xbar[r], d[r]);
+        column_stats<R>(col, p.n, nf, xbar[r], d[r], z[r]);
     }
-    accD += VEC ? (double)((d[0] + d[W > 1 ? 1 : 0]) + (d[W > 2 ? 2 : 0] + d[W > 3 ? 3 : 0])) : (double)d[0];
+    const bool d_ok = dev_usable<W>(d, z);
+    if (d_ok) accD += (double)group_sum<W>(d);
+    bool l_ok = true;
     if (LOSS) {
         const typename G::T hv = reinterpret_cast<const typename G::T*>(p.h)[q];
         const typename G::T cv = reinterpret_cast<const typename G::T*>(p.c)[q];
-        float l[W];
+        float l[W], hs[W], ts[W];
 #pragma unroll
         for (int r = 0; r < W; ++r) {
-            const float t = xbar[r] - G::lane(cv, r);
-            l[r] = (G::lane(hv, r) * t) * t;
+            hs[r] = G::lane(hv, r);
+            ts[r] = xbar[r] - G::lane(cv, r);
+            l[r] = (hs[r] * ts[r]) * ts[r];
         }
-        accL += VEC ? (double)((l[0] + l[W > 1 ? 1 : 0]) + (l[W > 2 ? 2 : 0] + l[W > 3 ? 3 : 0])) : (double)l[0];
+        l_ok = loss_usable<W>(l, hs, ts);
+        if (d_ok && l_ok) accL += (double)group_sum<W>(l);
     }
-    if (WRITE) {
+    if (WRITE && d_ok) {
         const typename G::T out = G::make(xbar);
 #pragma unroll
         for (int i = 0; i < R; ++i)
             if (i < p.n) reinterpret_cast<typename G::T*>(p.x + (int64_t)i * p.P)[q] = out;
     }
+    return d_ok && l_ok;
+}
+
+// Second pass over a thread's column groups, run only by threads for which finish_group returned
+// false.  The same fp32 arithmetic on x decides again.  A group whose d was usable was added (and
+// written back: its columns now all equal their mean, which averaging leaves unchanged, so d is
+// usable again and the mean and loss terms are the same); only a loss finish_group left out is
+// added here.  A group whose d was refused is still unchanged in x; it is redone here column by
+// column, with fp64 where a column needs it, and written back.
+template <bool VEC, bool LOSS, bool WRITE>
+__device__ void redo_group(const AvgParams& p, int64_t q, float nf, double& accD, double& accL)
+{
+    using G = ColumnGroup<VEC>;
+    constexpr int W = G::W;
+    float xbar[W], d[W], z[W], l[W], hs[W], ts[W];
+    for (int r = 0; r < W; ++r) {
+        const int64_t j = W * q + r;
+        column_stats_global(p.x, p.P, j, p.n, nf, xbar[r], d[r], z[r]);
+        if (LOSS) {
+            hs[r] = p.h[j];
+            ts[r] = xbar[r] - p.c[j];
+            l[r] = (hs[r] * ts[r]) * ts[r];
+        }
+    }
+    const bool d_ok = dev_usable<W>(d, z);
+    const bool l_ok = !LOSS || loss_usable<W>(l, hs, ts);
+    if (d_ok && l_ok) return;
+    for (int r = 0; r < W; ++r) {
+        const int64_t j = W * q + r;
+        if (!d_ok) accD += checked_sq_dev<0>([&](int i) { return p.x[(int64_t)i * p.P + j]; }, p.n, xbar[r], d[r]);
+        if (LOSS) accL += checked_loss_term(p.h[j], xbar[r], p.c[j]);
+    }
+    if (WRITE && !d_ok)
+        for (int r = 0; r < W; ++r)
+            for (int i = 0; i < p.n; ++i) p.x[(int64_t)i * p.P + W * q + r] = xbar[r];
 }
 
 // Persistent grid over column groups; each thread keeps the n replica values of U groups in
 // registers (NMAX >= n), so the loads of U groups are in flight together.  NMAX = 0: any n,
-// values re-read per pass.  The block partials are added by the last block to finish, in
+// values re-read per pass, fp64 inline where a column needs it.  The block partials are added by the last block to finish, in
 // block order, so the sums do not depend on which block finishes last.
 template <int NMAX, int U, bool VEC, bool LOSS, bool WRITE>
 __global__ void __launch_bounds__(kThreads, (NMAX >= 32 ? 1 : 2)) average_kernel(const AvgParams p)
@@ -225,6 +299,7 @@ __global__ void __launch_bounds__(kThreads, (NMAX >= 32 ? 1 : 2)) average_kernel
     __shared__ unsigned int ticket;
     const float nf = (float)p.n;
     double accD = 0.0, accL = 0.0;
+    bool redo = false;  // finish_group refused a group of this thread
     const int64_t stride = (int64_t)gridDim.x * kThreads;
     for (int64_t q0 = (int64_t)blockIdx.x * kThreads + threadIdx.x; q0 < p.Q; q0 += U * stride) {
         if (NMAX > 0) {
@@ -242,29 +317,18 @@ __global__ void __launch_bounds__(kThreads, (NMAX >= 32 ? 1 : 2)) average_kernel
 #pragma unroll
             for (int u = 0; u < U; ++u) {
                 const int64_t q = q0 + u * stride;
-                if (q < p.Q) finish_group<R, VEC, LOSS, WRITE>(p, q, vals[u], nf, accD, accL);
+                if (q < p.Q) redo |= !finish_group<R, VEC, LOSS, WRITE>(p, q, vals[u], nf, accD, accL);
             }
         } else {
             const int64_t q = q0;
-            float xbar[G::W], d[G::W];
+            float xbar[G::W];
 #pragma unroll
-            for (int r = 0; r < G::W; ++r) column_stats_global(p.x, p.P, G::W * q + r, p.n, nf, xbar[r], d[r]);
-            double dsum = 0.0;
-            float fsum = 0.0f;
-            if (VEC) fsum = (d[0] + d[G::W > 1 ? 1 : 0]) + (d[G::W > 2 ? 2 : 0] + d[G::W > 3 ? 3 : 0]);
-            dsum = VEC ? (double)fsum : (double)d[0];
-            accD += dsum;
-            if (LOSS) {
-                const T hv = reinterpret_cast<const T*>(p.h)[q];
-                const T cv = reinterpret_cast<const T*>(p.c)[q];
-                float l[G::W];
-#pragma unroll
-                for (int r = 0; r < G::W; ++r) {
-                    const float t = xbar[r] - G::lane(cv, r);
-                    l[r] = (G::lane(hv, r) * t) * t;
-                }
-                accL += VEC ? (double)((l[0] + l[G::W > 1 ? 1 : 0]) + (l[G::W > 2 ? 2 : 0] + l[G::W > 3 ? 3 : 0]))
-                            : (double)l[0];
+            for (int r = 0; r < G::W; ++r) {
+                const int64_t j = G::W * q + r;
+                float d, z;
+                column_stats_global(p.x, p.P, j, p.n, nf, xbar[r], d, z);
+                accD += checked_sq_dev<0>([&](int i) { return p.x[(int64_t)i * p.P + j]; }, p.n, xbar[r], d);
+                if (LOSS) accL += checked_loss_term(p.h[j], xbar[r], p.c[j]);
             }
             if (WRITE) {
                 const T out = G::make(xbar);
@@ -272,6 +336,9 @@ __global__ void __launch_bounds__(kThreads, (NMAX >= 32 ? 1 : 2)) average_kernel
             }
         }
     }
+    if (NMAX > 0 && redo)
+        for (int64_t q = (int64_t)blockIdx.x * kThreads + threadIdx.x; q < p.Q; q += stride)
+            redo_group<VEC, LOSS, WRITE>(p, q, nf, accD, accL);
     const double bD = block_sum(accD, shared);
     const double bL = LOSS ? block_sum(accL, shared) : 0.0;
     if (threadIdx.x == 0) {
