@@ -291,7 +291,7 @@ __device__ void redo_group(const AvgParams& p, int64_t q, float nf, double& accD
 // values re-read per pass, fp64 inline where a column needs it.  The block partials are added by the last block to finish, in
 // block order, so the sums do not depend on which block finishes last.
 template <int NMAX, int U, bool VEC, bool LOSS, bool WRITE>
-__global__ void __launch_bounds__(kThreads, (NMAX >= 32 ? 1 : 2)) average_kernel(const AvgParams p)
+__global__ void __launch_bounds__(kThreads, (NMAX == 2 ? 4 : (NMAX >= 32 ? 1 : 2))) average_kernel(const AvgParams p)
 {
     using G = ColumnGroup<VEC>;
     using T = typename G::T;
@@ -417,22 +417,26 @@ int max_blocks_per_sm(Kernel kernel)
 
 using AvgKernel = void (*)(const AvgParams);
 
-template <int NMAX, int U>
+template <int NMAX, int U, int UL = U>
 AvgKernel pick_average_nmax(bool vec, bool loss, bool write)
 {
+    // UL: groups per thread of the variant with the loss (h and c take registers too)
     if (vec) {
         if (!write) return average_kernel<NMAX, U, true, false, false>;
-        return loss ? average_kernel<NMAX, U, true, true, true> : average_kernel<NMAX, U, true, false, true>;
+        return loss ? average_kernel<NMAX, UL, true, true, true> : average_kernel<NMAX, U, true, false, true>;
     }
     if (!write) return average_kernel<NMAX, U, false, false, false>;
-    return loss ? average_kernel<NMAX, U, false, true, true> : average_kernel<NMAX, U, false, false, true>;
+    return loss ? average_kernel<NMAX, UL, false, true, true> : average_kernel<NMAX, U, false, false, true>;
 }
 
-// Register-resident variants: NMAX replicas x U column groups per thread (NMAX * U <= 32 float4;
-// for n <= 2, 4 groups measured 15 % faster than 8).
+// Register-resident variants: NMAX replicas x U column groups per thread (NMAX * U <= 32 float4).
+// Resident blocks per SM (the register cap): 4 for n <= 2, 1 for n <= 32 and 2 otherwise.  With
+// two rows per column a thread has few bytes in flight, so n <= 2 takes 4 blocks of 4 groups:
+// measured 0.93 of the copy peak at P = 2^28, against 0.71 with 2 blocks.  Its loss variant takes
+// 2 groups, which fit the 64 registers of that cap without spilling.
 AvgKernel pick_average(int32_t n, bool vec, bool loss, bool write)
 {
-    if (n <= 2) return pick_average_nmax<2, 4>(vec, loss, write);
+    if (n <= 2) return pick_average_nmax<2, 4, 2>(vec, loss, write);
     if (n <= 4) return pick_average_nmax<4, 4>(vec, loss, write);
     if (n <= 8) return pick_average_nmax<8, 2>(vec, loss, write);
     if (n <= 16) return pick_average_nmax<16, 1>(vec, loss, write);
