@@ -203,8 +203,9 @@ int adpsgd_average_and_variance(adpsgd_ctx* ctx, double* D_out, double* loss_out
  * The first call on each device looks up the scratch array's device address
  * (cudaGetSymbolAddress).  Make that first call before any stream capture.  Every call uses the
  * same array, which keeps the last call's contents.  Each call clears the completion counter in
- * it on the stream before the launch, and writes every other slot before reading it.  Calls that overlap on the GPU (several host threads,
- * or streams that run concurrently) race on the array and must be serialised by the caller.
+ * it on the stream before the launch, and writes every other slot before reading it.  Calls that
+ * overlap on the GPU (several host threads, or streams that run concurrently) race on the array
+ * and must be serialised by the caller.
  * Errors: E_INVAL, E_ALIGN, E_TIMEOUT, E_CUDA. */
 int adpsgd_average_and_variance_static(float* x, const float* h, const float* c, int32_t n, int64_t P,
                                        double* D_out, double* loss_out, int64_t wait_timeout_ms, void* stream);

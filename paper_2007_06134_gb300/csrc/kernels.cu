@@ -288,8 +288,9 @@ __device__ void redo_group(const AvgParams& p, int64_t q, float nf, double& accD
 
 // Persistent grid over column groups; each thread keeps the n replica values of U groups in
 // registers (NMAX >= n), so the loads of U groups are in flight together.  NMAX = 0: any n,
-// values re-read per pass, fp64 inline where a column needs it.  The block partials are added by the last block to finish, in
-// block order, so the sums do not depend on which block finishes last.
+// values re-read per pass, fp64 inline where a column needs it.  The block partials are added
+// by the last block to finish, in block order, so the sums do not depend on which block
+// finishes last.
 template <int NMAX, int U, bool VEC, bool LOSS, bool WRITE>
 __global__ void __launch_bounds__(kThreads, (NMAX == 2 ? 4 : (NMAX >= 32 ? 1 : 2))) average_kernel(const AvgParams p)
 {
