@@ -322,7 +322,7 @@ def run_gpu(args, w):
     k2_gbs = k2_bytes / (k2_ms / 1000.0) / 1e9
     clock_summary = clocks.summary()
 
-    # end to end through the C ABI from pinned host buffers
+    # end to end through the C ABI from pinned host buffers (copies, run and read-back)
     e2e_value, h2d, d2h, e2e_phases = None, 0, 0, None
     if not args.no_e2e:
         x0h = torch.zeros((n, P), dtype=torch.float32).pin_memory()
@@ -339,15 +339,14 @@ def run_gpu(args, w):
         marks = [torch.cuda.Event(enable_timing=True) for _ in range(4)]
 
         def e2e_step():
+            # inputs in and the averaged parameters out through the library's transfer calls
             marks[0].record(stream)
-            xd.copy_(x0h, non_blocking=True)
-            vd.copy_(v0h, non_blocking=True)
-            hd.copy_(hh, non_blocking=True)
-            cd.copy_(ch, non_blocking=True)
+            for dst, src in ((xd, x0h), (vd, v0h), (hd, hh), (cd, ch)):
+                abi.adpsgd_copy_h2d(dst, src, stream=stream)
             marks[1].record(stream)
             abi.adpsgd_run(ctx_e2e, sched, abi.adpsgd_state_init(sched))
             marks[2].record(stream)
-            xout.copy_(xd, non_blocking=True)
+            abi.adpsgd_copy_d2h(xout, xd, stream=stream)
             marks[3].record(stream)
 
         e2e_step()

@@ -262,6 +262,24 @@ int adpsgd_noise_fill_f32(uint64_t seed, uint32_t tag, int32_t n, int64_t P, int
  * to nearest-even bf16.  out: device, raw bf16 bits.  Enqueued only.  Errors: as above. */
 int adpsgd_noise_fill_bf16(uint64_t seed, int32_t n, int64_t P, uint16_t* out, void* stream);
 
+/* Moving a run's inputs and results between host and device: the state x, v and the
+ * objective h, c in, the averaged parameters out.  The paper has no counterpart (it trains on
+ * one machine per replica); these carry the end-to-end path from host buffers.
+ *
+ * adpsgd_copy_h2d copies `bytes` from host memory src to device memory dst, and
+ * adpsgd_copy_d2h from device memory src to host memory dst, enqueued on `stream`.  When the
+ * host buffer is page-locked (cudaHostAlloc, cudaHostRegister, PyTorch pinned memory), the
+ * library's copy kernel moves the bytes through the buffer's mapped device address.  That
+ * holds its throughput when other work loads the host memory, where the copy engines slow
+ * down.  Any other host memory goes through cudaMemcpyAsync.  The device side must be device
+ * (or managed) memory.  Both pointers 16-byte aligned; bytes need not be a multiple of 16.
+ * bytes == 0 does nothing.  The caller keeps both buffers alive until the stream has passed
+ * the copy.
+ * Errors: E_INVAL (NULL pointer with bytes > 0, bytes < 0, the device side not device memory,
+ * the host side device memory), E_ALIGN, E_CUDA. */
+int adpsgd_copy_h2d(void* dst, const void* src, int64_t bytes, void* stream);
+int adpsgd_copy_d2h(void* dst, const void* src, int64_t bytes, void* stream);
+
 /* Device time of the kernels launched through ctx while cfg.time_kernels was set, summed from
  * CUDA events on ctx's stream since init or the last reset (waits for them, bounded), over the
  * timed launches only (every time_kernels-th); *_launches counts those timed launches.

@@ -90,6 +90,8 @@ _SIGS = {
     "adpsgd_philox_fill": (C.c_int, [C.c_uint64, C.c_uint32, C.c_int32, C.c_int64, C.c_int64, _P, _P]),
     "adpsgd_noise_fill_f32": (C.c_int, [C.c_uint64, C.c_uint32, C.c_int32, C.c_int64, C.c_int64, _P, _P]),
     "adpsgd_noise_fill_bf16": (C.c_int, [C.c_uint64, C.c_int32, C.c_int64, _P, _P]),
+    "adpsgd_copy_h2d": (C.c_int, [_P, _P, C.c_int64, _P]),
+    "adpsgd_copy_d2h": (C.c_int, [_P, _P, C.c_int64, _P]),
     "adpsgd_kernel_times": (C.c_int, [_P, C.POINTER(KernelTiming)]),
     "adpsgd_reset_kernel_times": (C.c_int, [_P]),
     "adpsgd_test_force_incomplete": (C.c_int, [_P, C.c_int32]),
@@ -323,6 +325,20 @@ def adpsgd_noise_fill_f32(seed: int, tag: int, n: int, P: int, k: int, out, stre
 def adpsgd_noise_fill_bf16(seed: int, n: int, P: int, out, stream=None) -> None:
     _check(load().adpsgd_noise_fill_bf16(seed & 0xFFFFFFFFFFFFFFFF, n, P, _ptr(out), _stream(stream)),
            "adpsgd_noise_fill_bf16")
+
+
+def _nbytes(t, nbytes):
+    return t.numel() * t.element_size() if nbytes is None else nbytes
+
+
+def adpsgd_copy_h2d(dst, src, nbytes: int | None = None, stream=None) -> None:
+    """Host tensor src -> device tensor dst (nbytes: all of src by default), enqueued on stream."""
+    _check(load().adpsgd_copy_h2d(_ptr(dst), _ptr(src), _nbytes(src, nbytes), _stream(stream)), "adpsgd_copy_h2d")
+
+
+def adpsgd_copy_d2h(dst, src, nbytes: int | None = None, stream=None) -> None:
+    """Device tensor src -> host tensor dst (nbytes: all of src by default), enqueued on stream."""
+    _check(load().adpsgd_copy_d2h(_ptr(dst), _ptr(src), _nbytes(src, nbytes), _stream(stream)), "adpsgd_copy_d2h")
 
 
 def adpsgd_kernel_times(ctx: Context):

@@ -52,6 +52,10 @@ cudaError_t launch_average(const AverageArgs& a, cudaStream_t stream);
 int average_grid(int32_t n, int64_t P, bool loss, bool write_back, int sms);
 int average_grid_max(int sms);
 
+// bytes from src to dst by a copy kernel on `stream`.  Both are device addresses (for host
+// memory: the mapped device address of a page-locked buffer), 16-byte aligned.
+cudaError_t launch_copy(void* dst, const void* src, int64_t bytes, int sms, cudaStream_t stream);
+
 // Fixed device scratch (no allocation): partial sums for up to static_scratch_max_blocks()
 // blocks, the two finished sums and the completion counter.  The first call on a device looks the address up.
 int static_scratch_max_blocks();

@@ -773,6 +773,67 @@ int adpsgd_noise_fill_bf16(uint64_t seed, int32_t n, int64_t P, uint16_t* out, v
     return e == cudaSuccess ? ADPSGD_OK : cuda_fail(e, "bf16 noise fill");
 }
 
+namespace {
+
+// The kind of memory p points into (cudaMemoryTypeUnregistered for plain host memory).
+cudaError_t memory_type(const void* p, cudaMemoryType* type)
+{
+    cudaPointerAttributes attr;
+    const cudaError_t e = cudaPointerGetAttributes(&attr, p);
+    if (e != cudaSuccess) return e;
+    *type = attr.type;
+    return cudaSuccess;
+}
+
+// One host <-> device copy: `host` is the host side, `device` the device side; to_device
+// gives the direction.
+int transfer(void* dst, const void* src, int64_t bytes, void* stream, bool to_device)
+{
+    if (bytes < 0 || (bytes > 0 && (dst == nullptr || src == nullptr))) return ADPSGD_E_INVAL;
+    if (bytes == 0) return ADPSGD_OK;
+    if (!aligned16(dst) || !aligned16(src)) return ADPSGD_E_ALIGN;
+    const void* host = to_device ? src : dst;
+    const void* device = to_device ? dst : src;
+    cudaMemoryType host_type, device_type;
+    cudaError_t e = memory_type(device, &device_type);
+    if (e == cudaSuccess) e = memory_type(host, &host_type);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaPointerGetAttributes");
+    if (device_type != cudaMemoryTypeDevice && device_type != cudaMemoryTypeManaged) {
+        g_last_error = "the device side of the copy is not device memory";
+        return ADPSGD_E_INVAL;
+    }
+    if (host_type == cudaMemoryTypeDevice) {
+        g_last_error = "the host side of the copy is device memory";
+        return ADPSGD_E_INVAL;
+    }
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    void* mapped = nullptr;
+    if (host_type == cudaMemoryTypeHost && cudaHostGetDevicePointer(&mapped, const_cast<void*>(host), 0) == cudaSuccess &&
+        aligned16(mapped)) {
+        int device_id = 0, sms = 0;
+        e = cudaGetDevice(&device_id);
+        if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, device_id);
+        if (e != cudaSuccess) return cuda_fail(e, "device query");
+        e = to_device ? adpsgd::launch_copy(dst, mapped, bytes, sms, s) : adpsgd::launch_copy(mapped, src, bytes, sms, s);
+        return e == cudaSuccess ? ADPSGD_OK : cuda_fail(e, "copy kernel");
+    }
+    cudaGetLastError();  // a failed cudaHostGetDevicePointer leaves no sticky error; clear the last one
+    e = cudaMemcpyAsync(dst, src, (size_t)bytes, to_device ? cudaMemcpyHostToDevice : cudaMemcpyDeviceToHost, s);
+    return e == cudaSuccess ? ADPSGD_OK : cuda_fail(e, "cudaMemcpyAsync");
+}
+
+}  // namespace
+
+int adpsgd_copy_h2d(void* dst, const void* src, int64_t bytes, void* stream)
+{
+    return transfer(dst, src, bytes, stream, true);
+}
+
+int adpsgd_copy_d2h(void* dst, const void* src, int64_t bytes, void* stream)
+{
+    return transfer(dst, src, bytes, stream, false);
+}
+
 int adpsgd_kernel_times(adpsgd_ctx* ctx, adpsgd_kernel_timing* out)
 {
     if (ctx == nullptr || out == nullptr) return ADPSGD_E_INVAL;

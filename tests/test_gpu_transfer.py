@@ -1,0 +1,113 @@
+"""Host <-> device transfers through the C ABI (adpsgd_copy_h2d / adpsgd_copy_d2h).
+
+Page-locked host buffers go through the library's copy kernel; other host memory through
+cudaMemcpyAsync.  Both must deliver every byte, including ragged tails, interior pointers of a
+pinned allocation, and empty copies.  Bad arguments are refused before anything is enqueued.
+A whole run fed and read back through these calls matches the oracle.
+"""
+import numpy as np
+import pytest
+
+from oracle import oracle as O
+from paper_2007_06134_gb300 import abi, inputs
+
+pytestmark = pytest.mark.gpu
+
+torch = pytest.importorskip("torch")
+DEV = "cuda:0"
+
+
+def _bytes(nbytes, seed, pinned):
+    g = torch.Generator().manual_seed(seed)
+    t = torch.randint(0, 256, (nbytes,), dtype=torch.uint8, generator=g)
+    return t.pin_memory() if pinned else t
+
+
+@pytest.mark.parametrize("pinned", [True, False])
+@pytest.mark.parametrize("nbytes", [0, 1, 15, 16, 17, 4096 + 3, (1 << 20) + 5, (64 << 20) + 7])
+def test_round_trip(nbytes, pinned):
+    src = _bytes(nbytes, nbytes, pinned)
+    dev = torch.full((nbytes + 64,), 0xAB, dtype=torch.uint8, device=DEV)
+    back = torch.zeros(nbytes + 64, dtype=torch.uint8)
+    back = back.pin_memory() if pinned else back
+    abi.adpsgd_copy_h2d(dev, src, nbytes)
+    abi.adpsgd_copy_d2h(back, dev, nbytes)
+    torch.cuda.synchronize()
+    assert torch.equal(dev[:nbytes].cpu(), src)
+    assert bool((dev[nbytes:] == 0xAB).all()), "wrote past the end"
+    assert torch.equal(back[:nbytes], src) and bool((back[nbytes:] == 0).all())
+
+
+def test_interior_pointers_of_a_pinned_allocation():
+    big = _bytes(1 << 22, 3, True)
+    dev = torch.zeros(1 << 22, dtype=torch.uint8, device=DEV)
+    for off, ln in [(16, 1000), (4096, 123457), ((1 << 21) + 48, (1 << 20) + 1)]:
+        abi.adpsgd_copy_h2d(dev[off:], big[off:], ln)
+    torch.cuda.synchronize()
+    for off, ln in [(16, 1000), (4096, 123457), ((1 << 21) + 48, (1 << 20) + 1)]:
+        assert torch.equal(dev[off:off + ln].cpu(), big[off:off + ln])
+    out = torch.zeros(1 << 22, dtype=torch.uint8).pin_memory()
+    abi.adpsgd_copy_d2h(out[32:], dev[4096:], 123457)
+    torch.cuda.synchronize()
+    assert torch.equal(out[32:32 + 123457], big[4096:4096 + 123457])
+
+
+def test_copies_are_stream_ordered():
+    s = torch.cuda.Stream()
+    src = torch.arange(1 << 20, dtype=torch.float32).pin_memory()
+    dev = torch.zeros(1 << 20, device=DEV)
+    out = torch.zeros(1 << 20, dtype=torch.float32).pin_memory()
+    with torch.cuda.stream(s):
+        abi.adpsgd_copy_h2d(dev, src, stream=s)
+        dev.mul_(2.0)
+        abi.adpsgd_copy_d2h(out, dev, stream=s)
+    s.synchronize()
+    assert torch.equal(out, 2.0 * src)
+
+
+def test_bad_arguments_are_refused():
+    host = torch.zeros(64, dtype=torch.uint8).pin_memory()
+    pageable = torch.zeros(64, dtype=torch.uint8)
+    dev = torch.zeros(64, dtype=torch.uint8, device=DEV)
+    cases = [
+        (abi.adpsgd_copy_h2d, (dev[4:], host, 16), abi.E_ALIGN),
+        (abi.adpsgd_copy_h2d, (dev, host[4:], 16), abi.E_ALIGN),
+        (abi.adpsgd_copy_h2d, (host, pageable, 16), abi.E_INVAL),   # device side is host memory
+        (abi.adpsgd_copy_h2d, (pageable, host, 16), abi.E_INVAL),
+        (abi.adpsgd_copy_d2h, (host, host, 16), abi.E_INVAL),
+        (abi.adpsgd_copy_d2h, (dev, dev, 16), abi.E_INVAL),          # host side is device memory
+        (abi.adpsgd_copy_h2d, (dev, host, -1), abi.E_INVAL),
+        (abi.adpsgd_copy_h2d, (None, host, 16), abi.E_INVAL),
+    ]
+    for fn, args, status in cases:
+        with pytest.raises(abi.AdpsgdError) as e:
+            fn(*args)
+        assert e.value.status == status, (fn.__name__, status, e.value.status)
+    abi.adpsgd_copy_h2d(None, None, 0)  # empty copy: nothing to check, nothing done
+    torch.cuda.synchronize()
+
+
+def test_run_fed_and_read_back_through_the_transfer_calls():
+    w = inputs.WORKLOADS["quadratic-n4-P1M"]
+    n, P, K = w.n, (1 << 16) + 12, 40
+    h, c = inputs.problem(w, P)
+    x, v = inputs.random_state(n, P, 11)
+    xh, vh = torch.from_numpy(x).pin_memory(), torch.from_numpy(v).pin_memory()
+    hh, ch = torch.from_numpy(h).pin_memory(), torch.from_numpy(c).pin_memory()
+    xd, vd = torch.empty((n, P), device=DEV), torch.empty((n, P), device=DEV)
+    hd, cd = torch.empty(P, device=DEV), torch.empty(P, device=DEV)
+    for d, s in ((xd, xh), (vd, vh), (hd, hh), (cd, ch)):
+        abi.adpsgd_copy_h2d(d, s)
+    cfg = abi.make_config(n, P, momentum=w.mu, weight_decay=w.wd, noise_sigma=w.sigma, seed=w.seed)
+    sched = abi.make_schedule(abi.ADPSGD, K, 4, K_s=10, lr0=w.lr0)
+    tr = abi.TraceBuffers(K + 1)
+    with abi.adpsgd_init(cfg, xd, vd, hd, cd) as ctx:
+        abi.adpsgd_run(ctx, sched, abi.adpsgd_state_init(sched), trace=tr)
+    xo = torch.empty((n, P), dtype=torch.float32).pin_memory()
+    abi.adpsgd_copy_d2h(xo, xd)
+    torch.cuda.synchronize()
+    spec = O.ScheduleSpec(kind=abi.ADPSGD, K=K, p_init=4, K_s=10, lr0=w.lr0)
+    otr = O.run(x, v, h, c, spec=spec, seed=w.seed, mu=w.mu, wd=w.wd, sigma=w.sigma)
+    g = tr.arrays()
+    assert np.array_equal(g["k"], otr.k) and np.array_equal(g["p"], otr.p)
+    assert np.array_equal(xo.numpy().view(np.uint32), x.view(np.uint32))
