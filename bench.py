@@ -41,6 +41,7 @@ METRIC = "avg+variance GB/s vs HBM peak; fused local-step replica-params/sec"
 UNIT = "replica-params/s"
 CPU_SAMPLE_COLUMNS = 1 << 20
 TIMING_PERIOD = 4  # kernel durations from CUDA events around every 4th launch of each kernel
+AVG_SAMPLES = 24  # timed standalone averaging launches
 CPU_SAMPLE_ITERS = 24
 
 
@@ -59,10 +60,12 @@ def measured_peaks():
 
 KERNEL_SOURCES = {
     # kernel -> (file, first line marker, end marker) of the source it is built from
-    "local_step_kernel": [("kernels.cu", "struct StepParams", "struct AvgParams"), ("noise.cuh", "", ""),
+    "local_step_kernel": [("kernels.cu", "struct StepParams", "// Averaging + variance"), ("noise.cuh", "", ""),
                           ("common.cuh", "", "")],
-    "average_kernel": [("kernels.cu", "struct AvgParams", "__global__ void __launch_bounds__(kThreads) philox_fill"),
-                       ("common.cuh", "", "")],
+    "average_kernel": [("kernels.cu", "// Averaging + variance", "__global__ void __launch_bounds__(kThreads) philox_fill"),
+                       ("average.cuh", "", ""), ("common.cuh", "", "")],
+    "sync_step_kernel": [("sync_step.cu", "", ""), ("average.cuh", "", ""), ("noise.cuh", "", ""),
+                         ("common.cuh", "", "")],
 }
 
 
@@ -267,9 +270,10 @@ def run_gpu(args, w):
     if w.noise == "bf16":
         noise = torch.empty((n, P), dtype=torch.int16, device=device)
         abi.adpsgd_noise_fill_bf16(w.seed, n, P, noise, stream)
+    fuse_sync = not args.no_sync_fusion
     cfg = abi.make_config(n, P, momentum=w.mu, weight_decay=w.wd, noise_sigma=w.sigma, seed=seed,
                           noise_mode=abi.NOISE_BF16 if noise is not None else abi.NOISE_PHILOX, want_loss=True,
-                          time_kernels=TIMING_PERIOD)
+                          time_kernels=TIMING_PERIOD, fuse_sync_step=fuse_sync)
     sched = schedule_for(abi, w)
     ctx = abi.adpsgd_init(cfg, xd, vd, hd, cd, noise, stream)
 
@@ -301,7 +305,7 @@ def run_gpu(args, w):
         for _ in range(args.steps):
             stats = one_run()
             rounds.append(stats.rounds)
-            launches += stats.local_step_launches + stats.average_launches  # one kernel each
+            launches += stats.local_step_launches + stats.average_launches + stats.sync_step_launches
         ev1.record(stream)
         torch.cuda.synchronize(device)
         barrier(pg, device)
@@ -317,10 +321,25 @@ def run_gpu(args, w):
     k1_bytes = 16 * n * P + 8 * P + (2 * n * P if noise is not None else 0)
     k1_ms = kt["local_step_ms"] / max(1, kt["local_step_launches"])
     k1_gbs = k1_bytes / (k1_ms / 1000.0) / 1e9
-    k2_bytes = 8 * n * P + 8 * P
-    k2_ms = kt["average_ms"] / max(1, kt["average_launches"])
-    k2_gbs = k2_bytes / (k2_ms / 1000.0) / 1e9
+    # The fused sync step moves the local step's bytes: the averaging adds none.
+    ks_ms = kt["sync_step_ms"] / kt["sync_step_launches"] if kt["sync_step_launches"] else None
+    ks_gbs = k1_bytes / (ks_ms / 1000.0) / 1e9 if ks_ms else None
     clock_summary = clocks.summary()
+
+    # The averaging kernel on its own, as the unfused path runs it: one launch after each local
+    # step, every launch timed (with fused sync steps the run above launches few of them).
+    k2_bytes = 8 * n * P + 8 * P
+    cfg_k2 = abi.make_config(n, P, momentum=w.mu, weight_decay=w.wd, noise_sigma=w.sigma, seed=seed,
+                             noise_mode=cfg.noise_mode, want_loss=True, time_kernels=1)
+    with abi.adpsgd_init(cfg_k2, xd, vd, hd, cd, noise, stream) as ctx_k2:
+        for r in range(AVG_SAMPLES + 2):
+            if r == 2:
+                abi.adpsgd_reset_kernel_times(ctx_k2)
+            abi.adpsgd_local_steps(ctx_k2, r, [w.lr0])
+            abi.adpsgd_average_and_variance(ctx_k2)
+        kt2 = dict(abi.adpsgd_kernel_times(ctx_k2))
+    k2_ms = kt2["average_ms"] / max(1, kt2["average_launches"])
+    k2_gbs = k2_bytes / (k2_ms / 1000.0) / 1e9
 
     # end to end through the C ABI from pinned host buffers (copies, run and read-back)
     e2e_value, h2d, d2h, e2e_phases = None, 0, 0, None
@@ -333,7 +352,7 @@ def run_gpu(args, w):
         h2d = 4 * (2 * n * P + 2 * P)
         d2h = 4 * n * P
         cfg_e2e = abi.make_config(n, P, momentum=w.mu, weight_decay=w.wd, noise_sigma=w.sigma, seed=seed,
-                                  noise_mode=cfg.noise_mode, want_loss=True)
+                                  noise_mode=cfg.noise_mode, want_loss=True, fuse_sync_step=fuse_sync)
         ctx_e2e = abi.adpsgd_init(cfg_e2e, xd, vd, hd, cd, noise, stream)  # set-up, outside the timed region
 
         marks = [torch.cuda.Event(enable_timing=True) for _ in range(4)]
@@ -449,8 +468,16 @@ def run_gpu(args, w):
                          "traffic": recorded_traffic("local_step_kernel", w.name)},
             "avg_variance": {"kernel": "average_kernel", "bound": "hbm", "achieved": k2_gbs,
                              "peak": peak, "unit": "GB/s", "frac": k2_gbs / peak, "bytes_per_launch": k2_bytes,
-                             "ms_per_launch": k2_ms, "launches": kt["average_launches"],
+                             "ms_per_launch": k2_ms, "launches": kt2["average_launches"],
+                             "timed": "alone, each launch right after a local step",
                              "traffic": recorded_traffic("average_kernel", w.name)},
+            "sync_step": None if ks_ms is None else {
+                "kernel": "sync_step_kernel", "bound": "hbm", "achieved": ks_gbs, "peak": peak, "unit": "GB/s",
+                "frac": ks_gbs / peak, "bytes_per_launch": k1_bytes, "ms_per_launch": ks_ms,
+                "launches": kt["sync_step_launches"], "average_launches_in_run": kt["average_launches"],
+                "traffic": recorded_traffic("sync_step_kernel", w.name),
+                "note": "the local step of each sync iteration fused with its averaging (x not written "
+                        "and read back in between); 16 n P + 8 P bytes, the local step's"},
             "local_step_rp_per_s": n * P / (k1_ms / 1000.0),
             "fused_intervals": fused,
             "comparison": comparison,
@@ -569,6 +596,8 @@ def main():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu", action="store_true")
     ap.add_argument("--no-fused", action="store_true", help="skip the fused-interval measurement")
+    ap.add_argument("--no-sync-fusion", action="store_true",
+                    help="run each sync iteration's local step and averaging as two kernels")
     ap.add_argument("--no-compare", action="store_true", help="skip the ADPSGD / CPSGD / FULLSGD comparison runs")
     ap.add_argument("--sweep", action="store_true", help="averaging-kernel sweep over n x P instead")
     ap.add_argument("--sweep-max-bytes", type=float, default=70e9)

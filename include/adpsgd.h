@@ -73,6 +73,14 @@ typedef struct {
                                 the sync's averaging, as ONE kernel that keeps x and v in registers
                                 between steps.  Results are bit-identical to the unfused path.  Valid
                                 only because the surrogate objective is separable per column. */
+    int32_t fuse_sync_step;  /* nonzero: in adpsgd_run's per-iteration path, the local step of each
+                                iteration that ends with a sync and that averaging run as ONE
+                                kernel (x is not written and read back in between: 17 instead of
+                                25 bytes per replica-param).  Bit-identical results (D and the
+                                loss up to the order of fp64 additions).  Valid for any objective
+                                whose gradient is computed per element in the step; nothing is
+                                carried across steps.  Used where n <= 16, P % 4 == 0 and every
+                                array is 16-byte aligned (bf16 noise: 8-byte); elsewhere ignored. */
 } adpsgd_config;
 
 /* Schedules (Algorithm 1: kind 0; Algorithm 2: kind 1; kind 2: a piecewise-constant period,
@@ -141,7 +149,8 @@ typedef struct {
     double fullsgd_wire_bytes_per_node; /* one P-fp32 allreduce per iteration (FULLSGD) */
     int64_t local_step_launches;     /* kernel launches issued by this call: local steps, */
     int64_t average_launches;        /* averagings, */
-    int64_t interval_launches;       /* and fused intervals (cfg.fuse_intervals) */
+    int64_t interval_launches;       /* fused intervals (cfg.fuse_intervals), */
+    int64_t sync_step_launches;      /* and fused sync steps (cfg.fuse_sync_step) */
 } adpsgd_stats;
 
 /* Device time of the kernels launched through a context, from CUDA events on its stream. */
@@ -152,6 +161,8 @@ typedef struct {
     int64_t average_launches;
     double interval_ms;
     int64_t interval_launches;
+    double sync_step_ms;
+    int64_t sync_step_launches;
 } adpsgd_kernel_timing;
 
 /* Create a context over caller-owned device arrays.

@@ -34,7 +34,7 @@ class Config(C.Structure):
     _fields_ = [("n", C.c_int32), ("noise_mode", C.c_int32), ("P", C.c_int64), ("momentum", C.c_float),
                 ("weight_decay", C.c_float), ("noise_sigma", C.c_float), ("want_loss", C.c_int32),
                 ("seed", C.c_uint64), ("wait_timeout_ms", C.c_int64), ("time_kernels", C.c_int32),
-                ("fuse_intervals", C.c_int32)]
+                ("fuse_intervals", C.c_int32), ("fuse_sync_step", C.c_int32)]
 
 
 class Schedule(C.Structure):
@@ -63,12 +63,13 @@ class Stats(C.Structure):
     _fields_ = [("rounds", C.c_int64), ("equiv_period", C.c_double), ("wire_bytes_per_node", C.c_double),
                 ("wire_bytes_total", C.c_double), ("fullsgd_wire_bytes_per_node", C.c_double),
                 ("local_step_launches", C.c_int64), ("average_launches", C.c_int64),
-                ("interval_launches", C.c_int64)]
+                ("interval_launches", C.c_int64), ("sync_step_launches", C.c_int64)]
 
 
 class KernelTiming(C.Structure):
     _fields_ = [("local_step_ms", C.c_double), ("local_step_launches", C.c_int64), ("average_ms", C.c_double),
-                ("average_launches", C.c_int64), ("interval_ms", C.c_double), ("interval_launches", C.c_int64)]
+                ("average_launches", C.c_int64), ("interval_ms", C.c_double), ("interval_launches", C.c_int64),
+                ("sync_step_ms", C.c_double), ("sync_step_launches", C.c_int64)]
 
 
 _P = C.c_void_p
@@ -161,9 +162,11 @@ def _stream(stream) -> int | None:
 
 
 def make_config(n, P, *, momentum=0.9, weight_decay=0.0, noise_sigma=1.0, seed=0, noise_mode=NOISE_PHILOX,
-                want_loss=True, wait_timeout_ms=60000, time_kernels=False, fuse_intervals=False) -> Config:
+                want_loss=True, wait_timeout_ms=60000, time_kernels=False, fuse_intervals=False,
+                fuse_sync_step=False) -> Config:
     return Config(n, noise_mode, P, momentum, weight_decay, noise_sigma, int(bool(want_loss)),
-                  seed & 0xFFFFFFFFFFFFFFFF, wait_timeout_ms, int(time_kernels), int(bool(fuse_intervals)))
+                  seed & 0xFFFFFFFFFFFFFFFF, wait_timeout_ms, int(time_kernels), int(bool(fuse_intervals)),
+                  int(bool(fuse_sync_step)))
 
 
 def make_schedule(kind, K, p_init, *, K_s=0, K_w=0, lo=0.7, hi=1.3, p_min=1, p_max=0, lr0=0.1, lr_factor=0.1,

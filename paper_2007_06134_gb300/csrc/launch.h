@@ -52,6 +52,32 @@ cudaError_t launch_average(const AverageArgs& a, cudaStream_t stream);
 int average_grid(int32_t n, int64_t P, bool loss, bool write_back, int sms);
 int average_grid_max(int sms);
 
+// The local step of a sync iteration fused with the averaging that ends it: the same results
+// as launch_local_step followed by launch_average (write-back, loss when h_loss is set), with
+// out[0] = D and out[1] = loss as there.  Needs sync_step_supported().
+constexpr int kSyncStepMaxReplicas = 16;
+struct SyncStepArgs {
+    float* x;
+    float* v;
+    const float* h;
+    const float* c;
+    const uint16_t* noise_bf16;  // nullptr: Philox noise
+    const PhiloxKeys* keys;
+    int32_t n;
+    int64_t P;
+    uint32_t k;
+    float gamma, mu, wd, sigma;
+    bool loss;
+    double* partials;  // 2 * grid doubles
+    double* out;       // 2 doubles
+    unsigned int* counter;
+    int grid;          // from sync_step_grid()
+};
+bool sync_step_supported(int32_t n, int64_t P, const void* x, const void* v, const void* h, const void* c,
+                         const void* noise_bf16);
+int sync_step_grid(int32_t n, int64_t P, bool bf16, bool loss, int sms);
+cudaError_t launch_sync_step(const SyncStepArgs& a, cudaStream_t stream);
+
 // bytes from src to dst by a copy kernel on `stream`.  Both are device addresses (for host
 // memory: the mapped device address of a page-locked buffer), 16-byte aligned.
 cudaError_t launch_copy(void* dst, const void* src, int64_t bytes, int sms, cudaStream_t stream);

@@ -63,12 +63,14 @@ struct adpsgd_ctx {
     double* d_var = nullptr;  // per-iteration variance slots (2 doubles each), grown on demand
     int64_t d_var_cap = 0;
     int grid_avg = 0, grid_avg_loss = 0, grid_var = 0, grid_interval = 0;
+    int grid_sync = 0;  // > 0: the fused sync step is available (cfg.fuse_sync_step and supported)
     // kernel timing
     std::vector<cudaEvent_t> free_events;
     std::vector<TimedLaunch> pending;
-    double ms[3] = {0.0, 0.0, 0.0};
-    int64_t launches[3] = {0, 0, 0};
-    int64_t timed_launches[3] = {0, 0, 0};
+    // per kernel kind: 0 local step, 1 averaging, 2 fused interval, 3 fused sync step
+    double ms[4] = {0.0, 0.0, 0.0, 0.0};
+    int64_t launches[4] = {0, 0, 0, 0};
+    int64_t timed_launches[4] = {0, 0, 0, 0};
     bool force_incomplete = false;
 };
 
@@ -277,6 +279,39 @@ int interval(adpsgd_ctx* ctx, int64_t k0, int32_t m, const float* gamma, bool av
     return ADPSGD_OK;
 }
 
+// Enqueue the local step of iteration k fused with the averaging that ends it (needs
+// ctx->grid_sync > 0), the copy of the two sums into ctx->h_out, and ctx->done.
+int sync_step_enqueue(adpsgd_ctx* ctx, int64_t k, float gamma, bool loss)
+{
+    adpsgd::SyncStepArgs a;
+    a.x = ctx->x;
+    a.v = ctx->v;
+    a.h = ctx->h;
+    a.c = ctx->c;
+    a.noise_bf16 = ctx->noise;
+    a.keys = &ctx->keys;
+    a.n = ctx->cfg.n;
+    a.P = ctx->cfg.P;
+    a.k = (uint32_t)k;
+    a.gamma = gamma;
+    a.mu = ctx->cfg.momentum;
+    a.wd = ctx->cfg.weight_decay;
+    a.sigma = ctx->cfg.noise_sigma;
+    a.loss = loss;
+    a.partials = ctx->d_partials;
+    a.out = ctx->d_out;
+    a.counter = reinterpret_cast<unsigned int*>(ctx->d_out + 2);
+    a.grid = ctx->grid_sync;
+    int st = timed(ctx, 3, [&] { return adpsgd::launch_sync_step(a, ctx->stream); }, "sync step");
+    if (st != ADPSGD_OK) return st;
+    cudaError_t e = cudaMemcpyAsync(ctx->h_out, ctx->d_out, 2 * sizeof(double), cudaMemcpyDeviceToHost,
+                                    ctx->stream);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaMemcpyAsync");
+    e = cudaEventRecord(ctx->done, ctx->stream);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaEventRecord");
+    return ADPSGD_OK;
+}
+
 int check_schedule(const adpsgd_schedule* s)
 {
     if (s == nullptr) return ADPSGD_E_INVAL;
@@ -423,6 +458,8 @@ int adpsgd_init(const adpsgd_config* cfg, float* x, float* v, const float* h, co
     ctx->grid_avg_loss = adpsgd::average_grid(cfg->n, cfg->P, true, true, ctx->sms);
     ctx->grid_var = adpsgd::average_grid(cfg->n, cfg->P, false, false, ctx->sms);
     if (cfg->fuse_intervals) ctx->grid_interval = adpsgd::interval_grid(cfg->n, cfg->P, ctx->sms);
+    if (cfg->fuse_sync_step && adpsgd::sync_step_supported(cfg->n, cfg->P, x, v, h, c, ctx->noise))
+        ctx->grid_sync = adpsgd::sync_step_grid(cfg->n, cfg->P, ctx->noise != nullptr, cfg->want_loss != 0, ctx->sms);
     const int max_grid = std::max(adpsgd::average_grid_max(ctx->sms), adpsgd::interval_grid_max(ctx->sms));
     const size_t partial_bytes = 2 * sizeof(double) * (size_t)max_grid;
     e = cudaMalloc(reinterpret_cast<void**>(&ctx->d_partials), partial_bytes);
@@ -577,8 +614,7 @@ int adpsgd_run(adpsgd_ctx* ctx, const adpsgd_schedule* sched, adpsgd_state* stat
         }
         return local_step(ctx, k, gamma_of(sched, k));
     };
-    const int64_t launches0[2] = {ctx->launches[0], ctx->launches[1]};
-    const int64_t launches_fused0 = ctx->launches[2];
+    const int64_t launches0[4] = {ctx->launches[0], ctx->launches[1], ctx->launches[2], ctx->launches[3]};
     bool launched_ahead = false;  // the local step of iteration k is already enqueued
     if (ctx->cfg.fuse_intervals) {
         // One kernel per stretch of iterations up to and including the next sync (at most
@@ -625,15 +661,26 @@ int adpsgd_run(adpsgd_ctx* ctx, const adpsgd_schedule* sched, adpsgd_state* stat
         }
     }
     for (int64_t k = state->k_next; k < stop; ++k) {
-        if (!launched_ahead) {
-            st = step(k);
-            if (st != ADPSGD_OK) return st;
+        // Whether iteration k ends with a sync depends only on the schedule state, not on the
+        // step, so it is known before the step is enqueued.
+        // If enqueuing fails, the state goes back to the start of iteration k.
+        const adpsgd_state before = *state;
+        const bool sync = sync_after(sched, state, k);
+        if (sync && !launched_ahead && ctx->grid_sync > 0) {
+            // the step and the averaging as one kernel
+            if (track && k < trace->var_cap) st = variance_into_slot(ctx, k);
+            if (st == ADPSGD_OK) st = sync_step_enqueue(ctx, k, gamma_of(sched, k), loss);
+        } else {
+            if (!launched_ahead) st = step(k);
+            if (st == ADPSGD_OK && sync) st = average_enqueue(ctx, true, loss);
+        }
+        if (st != ADPSGD_OK) {
+            *state = before;
+            return st;
         }
         launched_ahead = false;
         state->k_next = k + 1;
-        if (!sync_after(sched, state, k)) continue;
-        st = average_enqueue(ctx, true, loss);
-        if (st != ADPSGD_OK) return st;
+        if (!sync) continue;
         // Whatever the rule decides, iteration k + 1 starts with a local step (p >= 1), so it is
         // enqueued behind the averaging before the host waits for S: the GPU stays busy while
         // the scalars travel to the host and the rule runs.
@@ -684,7 +731,8 @@ int adpsgd_run(adpsgd_ctx* ctx, const adpsgd_schedule* sched, adpsgd_state* stat
         wire(ctx->cfg.n, ctx->cfg.P, state->k_next, false, &stats->fullsgd_wire_bytes_per_node, &total);
         stats->local_step_launches = ctx->launches[0] - launches0[0];
         stats->average_launches = ctx->launches[1] - launches0[1];
-        stats->interval_launches = ctx->launches[2] - launches_fused0;
+        stats->interval_launches = ctx->launches[2] - launches0[2];
+        stats->sync_step_launches = ctx->launches[3] - launches0[3];
     }
     return ADPSGD_OK;
 }
@@ -846,6 +894,8 @@ int adpsgd_kernel_times(adpsgd_ctx* ctx, adpsgd_kernel_timing* out)
     out->average_launches = ctx->timed_launches[1];
     out->interval_ms = ctx->ms[2];
     out->interval_launches = ctx->timed_launches[2];
+    out->sync_step_ms = ctx->ms[3];
+    out->sync_step_launches = ctx->timed_launches[3];
     return ADPSGD_OK;
 }
 
@@ -856,8 +906,8 @@ int adpsgd_reset_kernel_times(adpsgd_ctx* ctx)
         int st = harvest_times(ctx);
         if (st != ADPSGD_OK) return st;
     }
-    ctx->ms[0] = ctx->ms[1] = ctx->ms[2] = 0.0;
-    ctx->timed_launches[0] = ctx->timed_launches[1] = ctx->timed_launches[2] = 0;
+    ctx->ms[0] = ctx->ms[1] = ctx->ms[2] = ctx->ms[3] = 0.0;
+    ctx->timed_launches[0] = ctx->timed_launches[1] = ctx->timed_launches[2] = ctx->timed_launches[3] = 0;
     return ADPSGD_OK;
 }
 

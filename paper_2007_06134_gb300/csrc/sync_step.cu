@@ -1,0 +1,151 @@
+// sync_step.cu -- the local step of a sync iteration fused with the averaging that ends it
+// (Algorithm 2: the last "updating parameter variables locally" of an interval, then the
+// averaging and S_k).  Each thread owns one float4 column group of all n replicas: it loads x,
+// v (and h, c once), applies the local step to every replica in registers with the same
+// operations as local_step_kernel, writes v, and then averages the new x with the same
+// operations as average_kernel (average.cuh).  Per replica-param that moves 16 B (+8/n) instead
+// of the 25 B of the two kernels run one after the other, since x is not written and read
+// back in between.  Nothing here depends on the objective being separable across steps: only
+// the update of one iteration is fused with the averaging that follows it.
+#include <cuda_runtime.h>
+
+#include <cstdint>
+
+#include "average.cuh"
+#include "common.cuh"
+#include "launch.h"
+#include "noise.cuh"
+
+namespace adpsgd {
+namespace {
+
+struct SyncStepParams {
+    AvgParams avg;          // x, h, c, P, Q = P / 4, n, partials, out, counter
+    float* v;
+    const uint16_t* noise;  // pre-materialised bf16 noise [n, P], or nullptr (Philox)
+    uint32_t k;
+    float gamma, mu, wd, sigma;
+    PhiloxKeys keys;
+};
+
+// Register cap: 128 per thread (2 blocks of 256 per SM) up to 8 replicas, 255 for 16.  One
+// thread per column group, no lane exchange: splitting a group's replicas over two lanes (and
+// swapping halves by shuffles) measured 10 % slower.
+template <int NMAX, bool BF16, bool LOSS>
+__global__ void __launch_bounds__(kThreads, (NMAX >= 16 ? 1 : 2)) sync_step_kernel(const SyncStepParams p)
+{
+    const AvgParams& a = p.avg;
+    const float nf = (float)a.n;
+    const bool wd = p.wd != 0.0f;
+    double accD = 0.0, accL = 0.0;
+    bool redo = false;
+    const int64_t stride = (int64_t)gridDim.x * kThreads;
+    for (int64_t q = (int64_t)blockIdx.x * kThreads + threadIdx.x; q < a.Q; q += stride) {
+        float4 xv[NMAX], vv[NMAX];
+        uint2 nb[NMAX];
+        const float4 hv = __ldg(reinterpret_cast<const float4*>(a.h) + q);
+        const float4 cv = __ldg(reinterpret_cast<const float4*>(a.c) + q);
+#pragma unroll
+        for (int i = 0; i < NMAX; ++i)
+            if (i < a.n) {
+                const int64_t row = (int64_t)i * a.P;
+                xv[i] = reinterpret_cast<const float4*>(a.x + row)[q];
+                vv[i] = reinterpret_cast<const float4*>(p.v + row)[q];
+                if (BF16) nb[i] = __ldg(reinterpret_cast<const uint2*>(p.noise + row) + q);
+            }
+#pragma unroll
+        for (int i = 0; i < NMAX; ++i)
+            if (i < a.n) {
+                const float4 z = BF16 ? make_float4(bf16_bits_to_float(nb[i].x & 0xFFFFu),
+                                                    __uint_as_float(nb[i].x & 0xFFFF0000u),
+                                                    bf16_bits_to_float(nb[i].y & 0xFFFFu),
+                                                    __uint_as_float(nb[i].y & 0xFFFF0000u))
+                                      : normals4(p.keys, (uint32_t)q, (uint32_t)i, p.k, 0u);
+                if (wd) {
+                    sgd_update<true>(xv[i].x, vv[i].x, hv.x, cv.x, z.x, p.gamma, p.mu, p.wd, p.sigma);
+                    sgd_update<true>(xv[i].y, vv[i].y, hv.y, cv.y, z.y, p.gamma, p.mu, p.wd, p.sigma);
+                    sgd_update<true>(xv[i].z, vv[i].z, hv.z, cv.z, z.z, p.gamma, p.mu, p.wd, p.sigma);
+                    sgd_update<true>(xv[i].w, vv[i].w, hv.w, cv.w, z.w, p.gamma, p.mu, p.wd, p.sigma);
+                } else {
+                    sgd_update<false>(xv[i].x, vv[i].x, hv.x, cv.x, z.x, p.gamma, p.mu, p.wd, p.sigma);
+                    sgd_update<false>(xv[i].y, vv[i].y, hv.y, cv.y, z.y, p.gamma, p.mu, p.wd, p.sigma);
+                    sgd_update<false>(xv[i].z, vv[i].z, hv.z, cv.z, z.z, p.gamma, p.mu, p.wd, p.sigma);
+                    sgd_update<false>(xv[i].w, vv[i].w, hv.w, cv.w, z.w, p.gamma, p.mu, p.wd, p.sigma);
+                }
+                reinterpret_cast<float4*>(p.v + (int64_t)i * a.P)[q] = vv[i];
+            }
+        redo |= !finish_group<NMAX, true, LOSS, true, true>(a, q, xv, nf, accD, accL);
+    }
+    if (redo)
+        for (int64_t q = (int64_t)blockIdx.x * kThreads + threadIdx.x; q < a.Q; q += stride)
+            redo_group<true, LOSS, true>(a, q, nf, accD, accL);
+    finish_sums<LOSS>(a, accD, accL);
+}
+
+using SyncStepKernel = void (*)(const SyncStepParams);
+
+template <int NMAX>
+SyncStepKernel pick_nmax(bool bf16, bool loss)
+{
+    if (bf16) return loss ? sync_step_kernel<NMAX, true, true> : sync_step_kernel<NMAX, true, false>;
+    return loss ? sync_step_kernel<NMAX, false, true> : sync_step_kernel<NMAX, false, false>;
+}
+
+SyncStepKernel pick(int32_t n, bool bf16, bool loss)
+{
+    if (n <= 2) return pick_nmax<2>(bf16, loss);
+    if (n <= 4) return pick_nmax<4>(bf16, loss);
+    if (n <= 8) return pick_nmax<8>(bf16, loss);
+    return pick_nmax<16>(bf16, loss);
+}
+
+}  // namespace
+
+bool sync_step_supported(int32_t n, int64_t P, const void* x, const void* v, const void* h, const void* c,
+                         const void* noise_bf16)
+{
+    auto al = [](const void* ptr, unsigned mask) { return (reinterpret_cast<uintptr_t>(ptr) & mask) == 0; };
+    return n >= 1 && n <= kSyncStepMaxReplicas && P % 4 == 0 && al(x, 15) && al(v, 15) && al(h, 15) && al(c, 15) &&
+           (noise_bf16 == nullptr || al(noise_bf16, 7));
+}
+
+int sync_step_grid(int32_t n, int64_t P, bool bf16, bool loss, int sms)
+{
+    int per_sm = 0;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, pick(n, bf16, loss), kThreads, 0) != cudaSuccess ||
+        per_sm < 1)
+        per_sm = 1;
+    const int64_t work = (P / 4 + kThreads - 1) / kThreads;
+    int64_t grid = (int64_t)per_sm * sms;
+    if (grid > work) grid = work;
+    if (grid < 1) grid = 1;
+    const int cap = average_grid_max(sms);
+    return (int)(grid > cap ? cap : grid);
+}
+
+cudaError_t launch_sync_step(const SyncStepArgs& s, cudaStream_t stream)
+{
+    SyncStepParams p;
+    p.avg.x = s.x;
+    p.avg.h = s.h;
+    p.avg.c = s.c;
+    p.avg.P = s.P;
+    p.avg.Q = s.P / 4;
+    p.avg.n = s.n;
+    p.avg.partials = s.partials;
+    p.avg.out = s.out;
+    p.avg.counter = s.counter;
+    p.v = s.v;
+    p.noise = s.noise_bf16;
+    p.k = s.k;
+    p.gamma = s.gamma;
+    p.mu = s.mu;
+    p.wd = s.wd;
+    p.sigma = s.sigma;
+    p.keys = *s.keys;
+    const SyncStepKernel kernel = pick(s.n, s.noise_bf16 != nullptr, s.loss);
+    kernel<<<(unsigned)s.grid, kThreads, 0, stream>>>(p);
+    return cudaGetLastError();
+}
+
+}  // namespace adpsgd

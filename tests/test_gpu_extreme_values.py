@@ -13,7 +13,7 @@ Each case runs through every averaging path:
 - the context entry point, with write-back and loss;
 - the variance-only entry point;
 - the entry point without a context;
-- the fused interval kernel inside a run.
+- the fused interval kernel and the fused sync step inside a run.
 The replica counts cover every register-resident variant and the any-n variant.
 """
 import numpy as np
@@ -123,22 +123,25 @@ def test_identical_replicas_give_exact_zero():
 
 
 @pytest.mark.parametrize("kind", ["tiny", "huge"])
-@pytest.mark.parametrize("fused", [False, True])
-def test_run_at_extreme_scales(kind, fused):
+@pytest.mark.parametrize("mode", ["unfused", "intervals", "sync_step"])
+def test_run_at_extreme_scales(kind, mode):
     # A short CPSGD run whose steps and syncs stay at the scale of the data: tiny values with tiny
     # noise (every sum subnormal), or huge values whose squares leave fp32.
-    n, P, K, p = 4, 1031, 6, 2
+    n, K, p = 4, 6, 2
+    P = 1032 if mode == "sync_step" else 1031  # the fused sync step takes P % 4 == 0 only
     x, h, c = _problem(n, P, kind, seed=5)
     scale = 1e-39 if kind == "tiny" else 1e30
     v = (0.1 * x).astype(F32)
     sigma, seed = scale, 0x5EED
     xd, vd = _dev(x), _dev(v)
-    cfg = abi.make_config(n, P, momentum=0.9, weight_decay=0.0, noise_sigma=sigma, seed=seed, fuse_intervals=fused)
+    cfg = abi.make_config(n, P, momentum=0.9, weight_decay=0.0, noise_sigma=sigma, seed=seed,
+                          fuse_intervals=mode == "intervals", fuse_sync_step=mode == "sync_step")
     sched = abi.make_schedule(abi.CPSGD, K, p, lr0=0.1)
     tr = abi.TraceBuffers(K + 1)
     with abi.adpsgd_init(cfg, xd, vd, _dev(h), _dev(c)) as ctx:
         stats = abi.adpsgd_run(ctx, sched, abi.adpsgd_state_init(sched), trace=tr)
-    assert (stats.interval_launches > 0) == fused
+    assert (stats.interval_launches > 0) == (mode == "intervals")
+    assert (stats.sync_step_launches > 0) == (mode == "sync_step")
     g = tr.arrays()
     spec = O.ScheduleSpec(kind=abi.CPSGD, K=K, p_init=p, lr0=0.1)
     otr = O.run(x, v, h, c, spec=spec, seed=seed, mu=0.9, wd=0.0, sigma=sigma)

@@ -1,0 +1,120 @@
+"""The fused sync step (cfg.fuse_sync_step): the local step of every iteration that ends with a
+sync, and that averaging, run as one kernel.  Whole runs must match the oracle exactly as the
+unfused path does (x, v, the mean and the schedule bit-exact; D and the loss within 1e-4), and
+match the unfused path itself.  Shapes the kernel does not take (n > 16, P not a multiple of 4)
+fall back to the separate kernels."""
+import numpy as np
+import pytest
+
+from oracle import oracle as O
+from paper_2007_06134_gb300 import abi, inputs
+
+pytestmark = pytest.mark.gpu
+
+torch = pytest.importorskip("torch")
+DEV = "cuda:0"
+REL = 1e-4
+
+
+def dev(a):
+    return torch.from_numpy(np.ascontiguousarray(a)).to(DEV)
+
+
+def host(t):
+    torch.cuda.synchronize()
+    return t.cpu().numpy()
+
+
+def rel(a, b):
+    return abs(a - b) / max(abs(b), 1e-300)
+
+
+def _run(n, P, K, kind, p, *, fused, wd=5e-4, bf16=False, loss=True, K_s=0, milestones=(), seed=3,
+         track=False, state=None):
+    w = inputs.WORKLOADS["resnet18-n8"]
+    h, c = inputs.draw_h(P, w.h_dist, seed), inputs.draw_c(P, 1.0, seed)
+    x, v = inputs.random_state(n, P, seed)
+    noise = O.noise_bf16(w.seed, n, P) if bf16 else None
+    xd, vd = dev(x), dev(v)
+    cfg = abi.make_config(n, P, momentum=0.9, weight_decay=wd, noise_sigma=0.8, seed=w.seed, want_loss=loss,
+                          noise_mode=abi.NOISE_BF16 if bf16 else abi.NOISE_PHILOX, fuse_sync_step=fused)
+    sched = abi.make_schedule(kind, K, p, K_s=K_s, lr0=0.1, milestones=milestones)
+    tr = abi.TraceBuffers(K + 1, var_cap=K if track else 0)
+    with abi.adpsgd_init(cfg, xd, vd, dev(h), dev(c), dev(noise.view(np.int16)) if bf16 else None) as ctx:
+        stats = abi.adpsgd_run(ctx, sched, abi.adpsgd_state_init(sched), trace=tr)
+    return dict(trace=tr.arrays(), stats=stats, x=host(xd), v=host(vd), inputs=(h, c, x, v, noise),
+                spec=O.ScheduleSpec(kind=kind, K=K, p_init=p, K_s=K_s, lr0=0.1, milestones=milestones),
+                wd=wd, seed=w.seed)
+
+
+def _against_oracle(r, loss=True):
+    h, c, x, v, noise = r["inputs"]
+    otr = O.run(x, v, h, c, spec=r["spec"], seed=r["seed"], mu=0.9, wd=r["wd"], sigma=0.8, noise=noise)
+    g = r["trace"]
+    assert np.array_equal(g["k"], otr.k) and np.array_equal(g["p"], otr.p) and np.array_equal(g["phase"], otr.phase)
+    for a, b in zip(g["S"], otr.S):
+        assert rel(a, b) < REL
+    if loss:
+        for a, b in zip(g["loss"], otr.loss):
+            assert rel(a, b) < REL
+    assert np.array_equal(r["x"].view(np.uint32), x.view(np.uint32))
+    assert np.array_equal(r["v"].view(np.uint32), v.view(np.uint32))
+
+
+@pytest.mark.parametrize("n", [1, 2, 3, 5, 8, 12, 16])
+@pytest.mark.parametrize("kind", [abi.ADPSGD, abi.CPSGD])
+def test_runs_match_the_oracle(n, kind):
+    P, K = 4096 + 4 * 37, 60
+    r = _run(n, P, K, kind, 4, fused=True, K_s=16 if kind == abi.ADPSGD else 0, milestones=(30,))
+    assert r["stats"].sync_step_launches > 0
+    assert r["stats"].sync_step_launches + r["stats"].average_launches == r["stats"].rounds
+    _against_oracle(r)
+
+
+@pytest.mark.parametrize("bf16,wd,loss", [(True, 0.0, True), (False, 0.0, False), (True, 5e-4, False)])
+def test_noise_modes_weight_decay_and_no_loss(bf16, wd, loss):
+    r = _run(8, 8192, 40, abi.ADPSGD, 3, fused=True, wd=wd, bf16=bf16, loss=loss, K_s=9)
+    assert r["stats"].sync_step_launches > 0
+    _against_oracle(r, loss=loss)
+
+
+def test_fused_equals_unfused_at_a_larger_size():
+    args = dict(n=8, P=(1 << 20) + 4 * 11, K=120, kind=abi.ADPSGD, p=4, K_s=30, milestones=(60, 90))
+    a = _run(fused=False, **args)
+    b = _run(fused=True, **args)
+    assert a["stats"].sync_step_launches == 0 and b["stats"].sync_step_launches > 0
+    for key in ("k", "p", "phase", "C2"):
+        assert np.array_equal(a["trace"][key], b["trace"][key])
+    assert np.array_equal(a["x"], b["x"]) and np.array_equal(a["v"], b["v"])
+    for s1, s2 in zip(a["trace"]["S"], b["trace"]["S"]):
+        assert rel(s1, s2) < 1e-6
+
+
+@pytest.mark.parametrize("n,P", [(17, 4096), (8, 4099), (4, 1)])
+def test_unsupported_shapes_fall_back(n, P):
+    r = _run(n, P, 30, abi.CPSGD, 3, fused=True)
+    assert r["stats"].sync_step_launches == 0 and r["stats"].average_launches == r["stats"].rounds
+    _against_oracle(r)
+
+
+def test_variance_record_with_fused_sync_steps():
+    a = _run(4, 4096, 40, abi.ADPSGD, 3, fused=False, K_s=10, track=True)
+    b = _run(4, 4096, 40, abi.ADPSGD, 3, fused=True, K_s=10, track=True)
+    assert b["stats"].sync_step_launches > 0
+    for s1, s2 in zip(a["trace"]["var"], b["trace"]["var"]):
+        assert rel(s1, s2) < 1e-6 or s1 == s2 == 0.0
+    assert np.array_equal(a["x"], b["x"])
+
+
+def test_kernel_times_count_the_sync_steps():
+    n, P, K = 4, 4096, 24
+    x, v = inputs.random_state(n, P, 1)
+    xd, vd = dev(x), dev(v)
+    z = torch.zeros(P, device=DEV)
+    cfg = abi.make_config(n, P, fuse_sync_step=True, time_kernels=1)
+    sched = abi.make_schedule(abi.CPSGD, K, 4, lr0=0.1)
+    with abi.adpsgd_init(cfg, xd, vd, z, z) as ctx:
+        st = abi.adpsgd_run(ctx, sched, abi.adpsgd_state_init(sched))
+        t = abi.adpsgd_kernel_times(ctx)
+    assert st.sync_step_launches == t["sync_step_launches"] == 6
+    assert t["local_step_launches"] == K - 6 and t["average_launches"] == 0 and t["sync_step_ms"] > 0
