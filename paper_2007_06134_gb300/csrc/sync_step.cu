@@ -29,8 +29,10 @@ struct SyncStepParams {
 };
 
 // Register cap: 128 per thread (2 blocks of 256 per SM) up to 8 replicas, 255 for 16.  One
-// thread per column group, no lane exchange: splitting a group's replicas over two lanes (and
-// swapping halves by shuffles) measured 10 % slower.
+// thread per column group.  Two other forms measured slower on resnet18-n8 (0.316 ms here):
+// splitting a group's replicas over two lanes that swap halves by shuffles (0.346 ms), and a
+// tiled form, with a thread per (group, replica) as in local_step_kernel and the averaging from a
+// shared-memory tile (0.350 ms).
 template <int NMAX, bool BF16, bool LOSS>
 __global__ void __launch_bounds__(kThreads, (NMAX >= 16 ? 1 : 2)) sync_step_kernel(const SyncStepParams p)
 {
@@ -113,8 +115,10 @@ int sync_step_grid(int32_t n, int64_t P, bool bf16, bool loss, int sms)
 {
     int per_sm = 0;
     if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, pick(n, bf16, loss), kThreads, 0) != cudaSuccess ||
-        per_sm < 1)
+        per_sm < 1) {
+        cudaGetLastError();
         per_sm = 1;
+    }
     const int64_t work = (P / 4 + kThreads - 1) / kThreads;
     int64_t grid = (int64_t)per_sm * sms;
     if (grid > work) grid = work;

@@ -83,11 +83,13 @@ def test_fused_equals_unfused_at_a_larger_size():
     a = _run(fused=False, **args)
     b = _run(fused=True, **args)
     assert a["stats"].sync_step_launches == 0 and b["stats"].sync_step_launches > 0
-    for key in ("k", "p", "phase", "C2"):
+    for key in ("k", "p", "phase"):
         assert np.array_equal(a["trace"][key], b["trace"][key])
     assert np.array_equal(a["x"], b["x"]) and np.array_equal(a["v"], b["v"])
-    for s1, s2 in zip(a["trace"]["S"], b["trace"]["S"]):
-        assert rel(s1, s2) < 1e-6
+    # S (and C2, built from it) differ only by the order of fp64 additions
+    for key in ("S", "C2"):
+        for s1, s2 in zip(a["trace"][key], b["trace"][key]):
+            assert rel(s1, s2) < 1e-6
 
 
 @pytest.mark.parametrize("n,P", [(17, 4096), (8, 4099), (4, 1)])
