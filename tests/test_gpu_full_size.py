@@ -44,9 +44,10 @@ def _sample_ranges(P, count=6):
     return ranges
 
 
-def _cfg(w, noise=False, fused=False):
+def _cfg(w, noise=False, mode="unfused"):
     return abi.make_config(w.n, w.P, momentum=w.mu, weight_decay=w.wd, noise_sigma=w.sigma, seed=w.seed,
-                           noise_mode=abi.NOISE_BF16 if noise else abi.NOISE_PHILOX, fuse_intervals=fused)
+                           noise_mode=abi.NOISE_BF16 if noise else abi.NOISE_PHILOX,
+                           fuse_intervals=mode == "intervals", fuse_sync_step=mode == "sync_step")
 
 
 def _oracle_noise_on_ranges(w, ranges):
@@ -58,10 +59,12 @@ def _oracle_noise_on_ranges(w, ranges):
     return noise
 
 
-@pytest.mark.parametrize("name,p,fused", [("resnet18-n8", 8, False), ("vgg16-n8", 8, False),
-                                          ("resnet50-n16-bf16noise", 4, False), ("resnet18-n8", 8, True),
-                                          ("resnet50-n16-bf16noise", 4, True)])
-def test_full_size_constant_period_run_on_sampled_columns(name, p, fused):
+# "sync_step" is the launch configuration bench.py times.
+@pytest.mark.parametrize("name,p,mode", [("resnet18-n8", 8, "unfused"), ("vgg16-n8", 8, "unfused"),
+                                         ("resnet50-n16-bf16noise", 4, "unfused"), ("resnet18-n8", 8, "intervals"),
+                                         ("resnet50-n16-bf16noise", 4, "intervals"), ("resnet18-n8", 8, "sync_step"),
+                                         ("vgg16-n8", 8, "sync_step"), ("resnet50-n16-bf16noise", 4, "sync_step")])
+def test_full_size_constant_period_run_on_sampled_columns(name, p, mode):
     w = inputs.WORKLOADS[name]
     bf16 = w.noise == "bf16"
     h, c = inputs.problem(w)
@@ -75,11 +78,15 @@ def test_full_size_constant_period_run_on_sampled_columns(name, p, fused):
         abi.adpsgd_noise_fill_bf16(w.seed, w.n, w.P, nd)
     sched = abi.make_schedule(abi.CPSGD, w.K, p, lr0=w.lr0, lr_factor=w.lr_factor, milestones=w.milestones)
     tr = abi.TraceBuffers(w.K)
-    with abi.adpsgd_init(_cfg(w, bf16, fused), xd, vd, _dev(h), _dev(c), nd) as ctx:
+    with abi.adpsgd_init(_cfg(w, bf16, mode), xd, vd, _dev(h), _dev(c), nd) as ctx:
         stats = abi.adpsgd_run(ctx, sched, abi.adpsgd_state_init(sched), trace=tr)
     torch.cuda.synchronize()
-    assert stats.rounds == w.K // p
-    assert (stats.interval_launches if fused else stats.local_step_launches) == (w.K // p if fused else w.K)
+    rounds = w.K // p
+    assert stats.rounds == rounds
+    launches = {"unfused": (w.K, rounds, 0, 0), "intervals": (0, 0, rounds, 0),
+                "sync_step": (w.K - rounds, 0, 0, rounds)}[mode]
+    assert (stats.local_step_launches, stats.average_launches, stats.interval_launches,
+            stats.sync_step_launches) == launches
     # oracle: the same run on the sampled columns only
     x = np.zeros((w.n, w.P), np.float32)
     v = np.zeros((w.n, w.P), np.float32)
@@ -119,7 +126,8 @@ def test_full_size_average_and_variance(name):
     assert np.array_equal(got.view(np.uint32), x.view(np.uint32))
 
 
-def test_full_size_adaptive_first_interval_and_rule_replay():
+@pytest.mark.parametrize("mode", ["unfused", "sync_step"])
+def test_full_size_adaptive_first_interval_and_rule_replay(mode):
     # resnet18-n8 at full size, Algorithm 2 (p_init 4, K_s 500): the first sync (after 4 local
     # steps from x0 = 0) against the oracle over all columns, and the whole trace against
     # Algorithm 2 replayed on the S values the run reported.
@@ -130,10 +138,11 @@ def test_full_size_adaptive_first_interval_and_rule_replay():
     sched = abi.make_schedule(abi.ADPSGD, w.K, w.p_init, K_s=w.K_s, lr0=w.lr0, lr_factor=w.lr_factor,
                               milestones=w.milestones)
     tr = abi.TraceBuffers(w.K)
-    with abi.adpsgd_init(_cfg(w), xd, vd, _dev(h), _dev(c)) as ctx:
+    with abi.adpsgd_init(_cfg(w, mode=mode), xd, vd, _dev(h), _dev(c)) as ctx:
         stats = abi.adpsgd_run(ctx, sched, abi.adpsgd_state_init(sched), trace=tr)
     t = tr.arrays()
     assert stats.rounds == len(t["k"]) and t["k"][0] == w.p_init - 1
+    assert (stats.sync_step_launches > 0) == (mode == "sync_step")
 
     x, v = inputs.zero_state(w.n, w.P)
     for k in range(w.p_init):
