@@ -232,6 +232,10 @@ int adpsgd_state_init(const adpsgd_schedule* sched, adpsgd_state* state);
  * Algorithm 1 when kind == ADPSGD_CPSGD): each iteration one local step with gamma_k, then
  * cnt += 1 and, when cnt reaches p, one averaging, S = D / n, and the period rule
  * (adpsgd_sched_on_sync).  Updates *state so that a later call resumes bit-identically.
+ * With cfg.fuse_intervals each stretch of steps up to a sync runs as one kernel; with
+ * cfg.fuse_sync_step the step of each iteration that ends with a sync, and that averaging, run
+ * as one kernel (except where that step was already enqueued ahead of the previous sync's wait,
+ * which happens only when p = 1).  Both give the same results as the separate kernels.
  * trace and stats may be NULL.  Blocks (bounded) at every sync.  Errors: E_INVAL (bad
  * schedule, K_s < p_init + K_w for kind 1, p < 1, trace->var with fuse_intervals), E_TIMEOUT,
  * E_CUDA.  After an error the state is not resumable (restore a checkpoint). */
