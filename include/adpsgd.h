@@ -235,7 +235,10 @@ int adpsgd_state_init(const adpsgd_schedule* sched, adpsgd_state* state);
  * With cfg.fuse_intervals each stretch of steps up to a sync runs as one kernel; with
  * cfg.fuse_sync_step the step of each iteration that ends with a sync, and that averaging, run
  * as one kernel (except where that step was already enqueued ahead of the previous sync's wait,
- * which happens only when p = 1).  Both give the same results as the separate kernels.
+ * which happens only when p = 1).  Both give the same x, v and schedule as the separate kernels;
+ * D, and so S, may differ in the last bits of its fp64 sum when the kernels' grids differ.  A
+ * call that resumes right after a sync with p = 1 may therefore fuse an iteration that an
+ * uninterrupted run ran as two kernels: x and v stay bit-identical, S may differ in its last bits.
  * trace and stats may be NULL.  Blocks (bounded) at every sync.  Errors: E_INVAL (bad
  * schedule, K_s < p_init + K_w for kind 1, p < 1, trace->var with fuse_intervals), E_TIMEOUT,
  * E_CUDA.  After an error the state is not resumable (restore a checkpoint). */
