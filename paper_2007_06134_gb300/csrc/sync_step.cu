@@ -29,11 +29,13 @@ struct SyncStepParams {
 };
 
 // Register cap: 128 per thread (2 blocks of 256 per SM) up to 8 replicas, 255 for 16.  One
-// thread per column group.  Two other forms measured slower on resnet18-n8 (0.316 ms here):
-// splitting a group's replicas over two lanes that swap halves by shuffles (0.346 ms), a tiled
-// form with a thread per (group, replica) as in local_step_kernel and the averaging from a
-// shared-memory tile (0.350 ms), and the step over the replicas in chunks of 4 under a runtime
-// loop, stashing the new x in shared memory, to shrink the unrolled code (0.336 ms).
+// thread per column group.  Other forms measured slower on resnet18-n8 (0.316 ms here):
+// - splitting a group's replicas over two lanes that swap halves by shuffles (0.346 ms);
+// - a tiled form, with a thread per (group, replica) as in local_step_kernel and the averaging
+//   from a shared-memory tile (0.350 ms);
+// - the step over the replicas in chunks of 4 under a runtime loop, stashing the new x in shared
+//   memory, to shrink the unrolled code (0.336 ms);
+// - this form capped at 80 registers for 3 blocks per SM, which spills (0.426 ms).
 template <int NMAX, bool BF16, bool LOSS>
 __global__ void __launch_bounds__(kThreads, (NMAX >= 16 ? 1 : 2)) sync_step_kernel(const SyncStepParams p)
 {
