@@ -70,14 +70,18 @@ KERNEL_SOURCES = {
 
 
 def kernel_source_digest(kernel: str) -> str:
-    """sha256 (16 hex) of the source text a kernel is compiled from."""
+    """sha256 (16 hex) of the code a kernel is compiled from, without comments and whitespace
+    (a comment edit does not invalidate a capture)."""
     import hashlib
+    import re
     h = hashlib.sha256()
     for fname, begin, end in KERNEL_SOURCES[kernel]:
         text = open(os.path.join(ROOT, "paper_2007_06134_gb300", "csrc", fname)).read()
         a = text.index(begin) if begin else 0
         b = text.index(end, a) if end else len(text)
-        h.update(text[a:b].encode())
+        code = re.sub(r"/\*.*?\*/", " ", text[a:b], flags=re.S)
+        code = re.sub(r"//[^\n]*", " ", code)
+        h.update(" ".join(code.split()).encode())
     return h.hexdigest()[:16]
 
 
