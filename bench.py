@@ -530,6 +530,62 @@ def run_sweep(args):
             del xd
 
 
+def run_sync_sweep(args):
+    """The fused sync step against the local step and the averaging it replaces, over n x P: a
+    CPSGD p = 2 run (every other iteration ends with a sync) with every launch timed, once with
+    fused sync steps and once with separate kernels.  Per point: each kernel's time, GB/s on its
+    algorithmic bytes, and the time saved per sync."""
+    import torch
+
+    from paper_2007_06134_gb300 import abi, inputs
+    peak, peak_kind = measured_peaks()
+    device = torch.device("cuda", 0)
+    stream = torch.cuda.current_stream(device)
+    w = inputs.WORKLOADS["resnet18-n8"]
+    # the shapes the fused step takes: up to 8 replicas with Philox noise, up to 16 with bf16 noise
+    for n, bf16 in ((2, False), (4, False), (8, False), (8, True), (16, True)):
+        for lp in (22, 24, 26):
+            P = 1 << lp
+            h, c = inputs.problem(w, P)
+            hd, cd = torch.from_numpy(h).to(device), torch.from_numpy(c).to(device)
+            xd = torch.zeros((n, P), dtype=torch.float32, device=device)
+            vd = torch.zeros_like(xd)
+            noise = None
+            if bf16:
+                noise = torch.empty((n, P), dtype=torch.int16, device=device)
+                abi.adpsgd_noise_fill_bf16(w.seed, n, P, noise, stream)
+            sched = abi.make_schedule(abi.CPSGD, 40, 2, lr0=w.lr0)
+            times = {}
+            for fused in (True, False):
+                cfg = abi.make_config(n, P, momentum=w.mu, weight_decay=w.wd, noise_sigma=w.sigma, seed=w.seed,
+                                      noise_mode=abi.NOISE_BF16 if bf16 else abi.NOISE_PHILOX,
+                                      time_kernels=1, fuse_sync_step=fused)
+                with abi.adpsgd_init(cfg, xd, vd, hd, cd, noise, stream) as ctx:
+                    abi.adpsgd_run(ctx, sched, abi.adpsgd_state_init(sched))
+                    abi.adpsgd_reset_kernel_times(ctx)
+                    abi.adpsgd_run(ctx, sched, abi.adpsgd_state_init(sched))
+                    t = abi.adpsgd_kernel_times(ctx)
+                if fused:
+                    times["sync_step"] = t["sync_step_ms"] / t["sync_step_launches"]
+                else:
+                    times["local_step"] = t["local_step_ms"] / t["local_step_launches"]
+                    times["average"] = t["average_ms"] / t["average_launches"]
+            step_bytes = 16 * n * P + 8 * P + (2 * n * P if bf16 else 0)
+            avg_bytes = 8 * n * P + 8 * P
+            line = {"sweep": "sync_step", "n": n, "P": P, "noise": "bf16" if bf16 else "philox",
+                    "peak": peak, "peak_kind": peak_kind,
+                    "sync_step_ms": times["sync_step"],
+                    "sync_step_frac": step_bytes / (times["sync_step"] / 1e3) / 1e9 / peak,
+                    "local_step_ms": times["local_step"],
+                    "local_step_frac": step_bytes / (times["local_step"] / 1e3) / 1e9 / peak,
+                    "average_ms": times["average"],
+                    "average_frac": avg_bytes / (times["average"] / 1e3) / 1e9 / peak,
+                    "saved_ms_per_sync": times["local_step"] + times["average"] - times["sync_step"],
+                    "l2": "x, v = %.0f MB" % (8 * n * P / 1e6)}
+            print(json.dumps(line), flush=True)
+            del xd, vd, noise
+
+
 def run_variance_traces(args):
     """The schedule study of Sec. IV on the strategies-n16 surrogate: constant periods, the four
     strategies' piecewise periods, the decreasing period of Sec. VI-B and Algorithm 2, each a whole
@@ -604,6 +660,8 @@ def main():
                     help="run each sync iteration's local step and averaging as two kernels")
     ap.add_argument("--no-compare", action="store_true", help="skip the ADPSGD / CPSGD / FULLSGD comparison runs")
     ap.add_argument("--sweep", action="store_true", help="averaging-kernel sweep over n x P instead")
+    ap.add_argument("--sync-sweep", action="store_true",
+                    help="fused sync step against the local step + averaging over n x P instead")
     ap.add_argument("--sweep-max-bytes", type=float, default=70e9)
     ap.add_argument("--variance-traces", action="store_true",
                     help="the schedule study of Sec. IV with per-iteration variance instead")
@@ -618,6 +676,8 @@ def main():
         return run_reference(args, w)
     if args.sweep:
         return run_sweep(args)
+    if args.sync_sweep:
+        return run_sync_sweep(args)
     if args.variance_traces:
         return run_variance_traces(args)
     return run_gpu(args, w)

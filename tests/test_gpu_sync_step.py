@@ -1,8 +1,9 @@
 """The fused sync step (cfg.fuse_sync_step): the local step of every iteration that ends with a
 sync, and that averaging, run as one kernel.  Whole runs must match the oracle exactly as the
 unfused path does (x, v, the mean and the schedule bit-exact; D and the loss within 1e-4), and
-match the unfused path itself.  Shapes the kernel does not take (n > 16, P not a multiple of 4)
-fall back to the separate kernels."""
+match the unfused path itself.  Shapes the kernel does not take fall back to the separate
+kernels: P not a multiple of 4, more than 8 replicas with Philox noise, more than 16 with the bf16
+noise tensor."""
 import numpy as np
 import pytest
 
@@ -61,11 +62,13 @@ def _against_oracle(r, loss=True):
     assert np.array_equal(r["v"].view(np.uint32), v.view(np.uint32))
 
 
-@pytest.mark.parametrize("n", [1, 2, 3, 5, 8, 12, 16])
+# n <= 8 with Philox noise; 9..16 replicas take the fused step with the bf16 noise tensor only.
+@pytest.mark.parametrize("n,bf16", [(1, False), (2, False), (3, False), (5, False), (8, False), (12, True),
+                                    (16, True)])
 @pytest.mark.parametrize("kind", [abi.ADPSGD, abi.CPSGD])
-def test_runs_match_the_oracle(n, kind):
+def test_runs_match_the_oracle(n, bf16, kind):
     P, K = 4096 + 4 * 37, 60
-    r = _run(n, P, K, kind, 4, fused=True, K_s=16 if kind == abi.ADPSGD else 0, milestones=(30,))
+    r = _run(n, P, K, kind, 4, fused=True, bf16=bf16, K_s=16 if kind == abi.ADPSGD else 0, milestones=(30,))
     assert r["stats"].sync_step_launches > 0
     assert r["stats"].sync_step_launches + r["stats"].average_launches == r["stats"].rounds
     _against_oracle(r)
@@ -92,7 +95,7 @@ def test_fused_equals_unfused_at_a_larger_size():
             assert rel(s1, s2) < 1e-6
 
 
-@pytest.mark.parametrize("n,P", [(17, 4096), (8, 4099), (4, 1)])
+@pytest.mark.parametrize("n,P", [(17, 4096), (8, 4099), (4, 1), (9, 4096), (16, 4096)])
 def test_unsupported_shapes_fall_back(n, P):
     r = _run(n, P, 30, abi.CPSGD, 3, fused=True)
     assert r["stats"].sync_step_launches == 0 and r["stats"].average_launches == r["stats"].rounds
