@@ -14,6 +14,10 @@
 //                      atomic ticket, no inter-block wait).  HBM-bound: 8 B per replica-param.
 //   *_fill kernels     the raw Philox stream, its fp32 normals, and the bf16 noise tensor.
 //
+// The averaging's per-group arithmetic (mean, squared deviations, loss, the fp32-range guard and
+// its second pass, the block sums) is in average.cuh, shared with sync_step_kernel
+// (sync_step.cu), which fuses a sync iteration's local step with its averaging.
+//
 // Every fp32 operation of the update, the mean and the generator is written out once and
 // compiled with -fmad=false, so results are bit-identical to any IEEE evaluation of the same
 // sequence.
