@@ -64,8 +64,8 @@ KERNEL_SOURCES = {
                           ("common.cuh", "", "")],
     "average_kernel": [("kernels.cu", "// Averaging + variance", "__global__ void __launch_bounds__(kThreads) philox_fill"),
                        ("average.cuh", "", ""), ("common.cuh", "", "")],
-    "sync_step_kernel": [("sync_step.cu", "", ""), ("average.cuh", "", ""), ("noise.cuh", "", ""),
-                         ("common.cuh", "", "")],
+    "sync_step_kernel": [("sync_step.cu", "struct SyncStepParams", "using SyncStepKernel"), ("average.cuh", "", ""),
+                         ("noise.cuh", "", ""), ("common.cuh", "", "")],
 }
 
 
