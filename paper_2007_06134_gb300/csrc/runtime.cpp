@@ -1,6 +1,7 @@
 // runtime.cpp -- host side of the C ABI in include/adpsgd.h: argument checks, the context,
 // the ADPSGD period rule (Algorithm 2), the step-size schedule, the run loop and the bounded
-// waits.  All device work goes through the kernels in kernels.cu on the caller's stream.
+// waits.  All device work goes through the library's kernels (kernels.cu, sync_step.cu,
+// interval.cu, transfer.cu) on the caller's stream.
 #include <cuda_runtime_api.h>
 
 #include <algorithm>
@@ -42,7 +43,7 @@ constexpr int64_t kMaxK = int64_t(1) << 32;  // the step index is one 32-bit Phi
 
 struct TimedLaunch {
     cudaEvent_t start, stop;
-    int kind;  // 0 local step, 1 averaging, 2 fused interval
+    int kind;  // 0 local step, 1 averaging, 2 fused interval, 3 fused sync step
 };
 
 struct adpsgd_ctx {
