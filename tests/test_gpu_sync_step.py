@@ -123,3 +123,31 @@ def test_kernel_times_count_the_sync_steps():
         t = abi.adpsgd_kernel_times(ctx)
     assert st.sync_step_launches == t["sync_step_launches"] == 6
     assert t["local_step_launches"] == K - 6 and t["average_launches"] == 0 and t["sync_step_ms"] > 0
+
+
+@pytest.mark.parametrize("split", [17, 20, 33])
+def test_resume_with_fused_sync_steps(split):
+    # One call against two calls split at iteration `split` (CPSGD p = 4: 20 ends right after a
+    # sync, 17 and 33 fall inside an interval): x, v and the schedule are bit-identical.
+    n, P, K = 8, 4096 + 64, 48
+    w = inputs.WORKLOADS["resnet18-n8"]
+    h, c = inputs.draw_h(P, w.h_dist, 4), inputs.draw_c(P, 1.0, 4)
+    x0, v0 = inputs.random_state(n, P, 4)
+    cfg = abi.make_config(n, P, momentum=0.9, weight_decay=5e-4, noise_sigma=0.8, seed=9, fuse_sync_step=True)
+    sched = abi.make_schedule(abi.CPSGD, K, 4, lr0=0.1)
+    out = []
+    for calls in ([K], [split, K]):
+        xd, vd = dev(x0), dev(v0)
+        tr = abi.TraceBuffers(K + 1)
+        with abi.adpsgd_init(cfg, xd, vd, dev(h), dev(c)) as ctx:
+            st = abi.adpsgd_state_init(sched)
+            for k_end in calls:
+                abi.adpsgd_run(ctx, sched, st, k_end=k_end, trace=tr)
+        out.append((host(xd), host(vd), tr.arrays(), st))
+    (xa, va, ta, sa), (xb, vb, tb, sb) = out
+    assert np.array_equal(xa.view(np.uint32), xb.view(np.uint32))
+    assert np.array_equal(va.view(np.uint32), vb.view(np.uint32))
+    assert np.array_equal(ta["k"], tb["k"]) and np.array_equal(ta["p"], tb["p"])
+    for s1, s2 in zip(ta["S"], tb["S"]):
+        assert rel(s1, s2) < 1e-12
+    assert (sa.k_next, sa.cnt, sa.p, sa.rounds) == (sb.k_next, sb.cnt, sb.p, sb.rounds)
