@@ -162,11 +162,16 @@ def test_full_size_adaptive_first_interval_and_rule_replay(mode):
     assert k_expect >= w.K
 
 
+def _cfg_big(n, P, mu, wd, sigma, seed, mode):
+    return abi.make_config(n, P, momentum=mu, weight_decay=wd, noise_sigma=sigma, seed=seed,
+                           fuse_sync_step=mode == "sync_step", fuse_intervals=mode == "intervals")
+
+
 def test_more_than_2_31_elements():
     # n P = 2^31 + 8 elements per array: the 64-bit index arithmetic of the local step, the
-    # averaging and the fused sync step, checked on columns on both sides of 2^30 and at the end
-    # (x and v bit-exact against the oracle).  About 26 GB of HBM; the host arrays are lazily
-    # zeroed, so only the sampled columns' pages are touched.
+    # averaging, the fused sync step and the fused interval, on columns on both sides of 2^30
+    # and at the end (x and v bit-exact against the oracle).  About 26 GB of HBM; the host arrays
+    # are lazily zeroed, so only the sampled columns' pages are touched.
     n, P = 2, (1 << 30) + 4
     ranges = [(0, 64), ((1 << 29) - 32, (1 << 29) + 32), ((1 << 30) - 32, (1 << 30) + 4)]
     gen = torch.Generator(device=DEV).manual_seed(31)
@@ -179,14 +184,14 @@ def test_more_than_2_31_elements():
         c[j0:j1] = cd[j0:j1].cpu().numpy()
     seed, mu, wd, sigma, lr = 77, 0.9, 5e-4, 0.5, 0.05
     sched = abi.make_schedule(abi.CPSGD, 4, 4, lr0=lr)
-    for fused in (False, True):
+    for mode in ("unfused", "sync_step", "intervals"):
         xd = torch.zeros((n, P), dtype=torch.float32, device=DEV)
         vd = torch.zeros_like(xd)
-        cfg = abi.make_config(n, P, momentum=mu, weight_decay=wd, noise_sigma=sigma, seed=seed,
-                              fuse_sync_step=fused)
-        with abi.adpsgd_init(cfg, xd, vd, hd, cd) as ctx:
+        with abi.adpsgd_init(_cfg_big(n, P, mu, wd, sigma, seed, mode), xd, vd, hd, cd) as ctx:
             st = abi.adpsgd_run(ctx, sched, abi.adpsgd_state_init(sched))
-        assert st.rounds == 1 and st.sync_step_launches == (1 if fused else 0)
+        assert st.rounds == 1
+        assert (st.sync_step_launches, st.interval_launches) == {"unfused": (0, 0), "sync_step": (1, 0),
+                                                                 "intervals": (0, 1)}[mode]
         x = np.zeros((n, P), np.float32)
         v = np.zeros((n, P), np.float32)
         for j0, j1 in ranges:
@@ -196,7 +201,7 @@ def test_more_than_2_31_elements():
             O.average_variance(x, h, c, j0, j1)
             gx = xd[:, j0:j1].cpu().numpy()
             gv = vd[:, j0:j1].cpu().numpy()
-            assert np.array_equal(gx.view(np.uint32), x[:, j0:j1].view(np.uint32)), (fused, j0)
-            assert np.array_equal(gv.view(np.uint32), v[:, j0:j1].view(np.uint32)), (fused, j0)
+            assert np.array_equal(gx.view(np.uint32), x[:, j0:j1].view(np.uint32)), (mode, j0)
+            assert np.array_equal(gv.view(np.uint32), v[:, j0:j1].view(np.uint32)), (mode, j0)
         del xd, vd
         torch.cuda.empty_cache()
