@@ -151,3 +151,29 @@ def test_resume_with_fused_sync_steps(split):
     for s1, s2 in zip(ta["S"], tb["S"]):
         assert rel(s1, s2) < 1e-12
     assert (sa.k_next, sa.cnt, sa.p, sa.rounds) == (sb.k_next, sb.cnt, sb.p, sb.rounds)
+
+
+@pytest.mark.parametrize("fused", [False, True])
+def test_noise_free_identical_replicas(fused):
+    # sigma = 0 from a shared start: the replicas stay identical, every sync reports D = 0 exactly
+    # (the exact-zero test, no fp64 path) and Algorithm 2 keeps p (0 is neither < 0.7 nor > 1.3
+    # times gamma C2 = 0).  x matches the oracle bit for bit.
+    n, P, K = 8, 4096, 40
+    w = inputs.WORKLOADS["resnet18-n8"]
+    h, c = inputs.draw_h(P, w.h_dist, 6), inputs.draw_c(P, 1.0, 6)
+    base, _ = inputs.random_state(1, P, 6)
+    x = np.repeat(base, n, axis=0)
+    v = np.zeros_like(x)
+    xd, vd = dev(x), dev(v)
+    cfg = abi.make_config(n, P, momentum=0.9, weight_decay=5e-4, noise_sigma=0.0, seed=1, fuse_sync_step=fused)
+    sched = abi.make_schedule(abi.ADPSGD, K, 3, K_s=9, lr0=0.1)
+    tr = abi.TraceBuffers(K + 1)
+    with abi.adpsgd_init(cfg, xd, vd, dev(h), dev(c)) as ctx:
+        st = abi.adpsgd_run(ctx, sched, abi.adpsgd_state_init(sched), trace=tr)
+    g = tr.arrays()
+    assert (st.sync_step_launches > 0) == fused
+    assert np.all(g["S"] == 0.0) and np.all(g["p"] == 3) and np.all(g["C2"] == 0.0)
+    spec = O.ScheduleSpec(kind=abi.ADPSGD, K=K, p_init=3, K_s=9, lr0=0.1)
+    otr = O.run(x, v, h, c, spec=spec, seed=1, mu=0.9, wd=5e-4, sigma=0.0)
+    assert np.array_equal(g["k"], otr.k) and np.all(otr.S == 0.0)
+    assert np.array_equal(host(xd).view(np.uint32), x.view(np.uint32))
