@@ -23,6 +23,8 @@
  *   - The period rule of Algorithm 2 (cnt, p, C_2; sampling phase k < K_s;
  *     +1 / -1 at 0.7 and 1.3) and Algorithm 1 as the constant-period case.
  *   - The bytes a ring allreduce would put on the wire per schedule.
+ *   - The same run on all host cores (OpenMP over fixed column chunks, the
+ *     fp64 partial sums added in chunk order), for full-size comparisons.
  *
  * Precision.  Parameters and momentum buffers are fp32 (the experiments ran
  * PyTorch 1.0 defaults); every fp32 operation below is separately rounded
@@ -299,13 +301,17 @@ void orc_local_step(int32_t n, int64_t P, int64_t j0, int64_t j1, float* x, floa
     for (int32_t i = 0; i < n; ++i) {
         float* xi = x + (int64_t)i * P;
         float* vi = v + (int64_t)i * P;
+        float zb[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+        int64_t block = -1;  /* the Philox block whose four normals zb holds */
         for (int64_t j = j0; j < j1; ++j) {
             float z;
             if (noise_bf16 != NULL) {
                 z = from_bf16(noise_bf16[(int64_t)i * P + j]);
             } else {
-                float zb[4];
-                normals_of_block(seed, 0u, (uint32_t)i, (uint32_t)k, (uint64_t)(j / 4), zb);
+                if (j / 4 != block) {
+                    block = j / 4;
+                    normals_of_block(seed, 0u, (uint32_t)i, (uint32_t)k, (uint64_t)block, zb);
+                }
                 z = zb[j % 4];
             }
             float diff = xi[j] - c[j];
@@ -355,11 +361,11 @@ void orc_average_variance(int32_t n, int64_t P, int64_t j0, int64_t j1, float* x
     if (loss != NULL) *loss += lsum;
 }
 
-/* Variance only (no write-back), for per-iteration diagnostics: D as above. */
-double orc_variance(int32_t n, int64_t P, const float* x)
+/* Variance only (no write-back) of columns [j0, j1), for per-iteration diagnostics: D as above. */
+double orc_variance_cols(int32_t n, int64_t P, int64_t j0, int64_t j1, const float* x)
 {
     double dsum = 0.0;
-    for (int64_t j = 0; j < P; ++j) {
+    for (int64_t j = j0; j < j1; ++j) {
         float base = x[j];
         float acc = 0.0f;
         for (int32_t i = 1; i < n; ++i) acc = acc + (x[(int64_t)i * P + j] - base);
@@ -371,6 +377,8 @@ double orc_variance(int32_t n, int64_t P, const float* x)
     }
     return dsum;
 }
+
+double orc_variance(int32_t n, int64_t P, const float* x) { return orc_variance_cols(n, P, 0, P, x); }
 
 /* ------------------------------------------------------------------------ */
 /* Schedules.                                                                */
@@ -521,6 +529,77 @@ int64_t orc_run(int32_t n, int64_t P, float* x, float* v, const float* h, const 
         }
         syncs = syncs + 1;
     }
+    return syncs;
+}
+
+/* ------------------------------------------------------------------------ */
+/* The same run on several host threads (OpenMP).  The columns are cut into  */
+/* fixed chunks of `chunk` columns, a multiple of 4 so that no Philox block  */
+/* is split; each thread runs the per-element code above on whole chunks.   */
+/* The fp64 partial sums of D and the loss (and of the per-iteration         */
+/* variance) are kept per chunk and added in chunk order, so the result does */
+/* not depend on the thread count.  x, v, the sync iterations, the periods   */
+/* and the phases equal orc_run's bit for bit; D and the loss differ from    */
+/* orc_run's only in the order of their fp64 additions.                      */
+/* Returns the number of syncs, or -1 if chunk is not a positive multiple    */
+/* of 4 or the partial sums cannot be allocated.                             */
+/* ------------------------------------------------------------------------ */
+int64_t orc_run_chunked(int32_t threads, int64_t chunk, int32_t n, int64_t P, float* x, float* v,
+                        const float* h, const float* c, const uint16_t* noise_bf16, uint64_t seed,
+                        float mu, float wd, float sigma, const orc_schedule* s, orc_state* st,
+                        int64_t k_begin, int64_t k_end, orc_trace* tr)
+{
+    if (chunk <= 0 || chunk % 4 != 0) return -1;
+    const int64_t nchunks = (P + chunk - 1) / chunk;
+    double* part = (double*)calloc((size_t)(2 * nchunks + 1), sizeof(double));
+    if (part == NULL) return -1;
+    double* partD = part;
+    double* partL = part + nchunks;
+    if (threads < 1) threads = 1;
+    int64_t syncs = 0;
+    for (int64_t k = k_begin; k < k_end; ++k) {
+        float gamma = orc_gamma(s, k);
+        if (tr != NULL && tr->var != NULL && k < tr->var_cap) {
+            #pragma omp parallel for num_threads(threads) schedule(static)
+            for (int64_t ch = 0; ch < nchunks; ++ch) {
+                const int64_t j1 = (ch + 1) * chunk < P ? (ch + 1) * chunk : P;
+                partD[ch] = orc_variance_cols(n, P, ch * chunk, j1, x);
+            }
+            double D = 0.0;
+            for (int64_t ch = 0; ch < nchunks; ++ch) D += partD[ch];
+            tr->var[k] = D / (double)n;
+        }
+        #pragma omp parallel for num_threads(threads) schedule(static)
+        for (int64_t ch = 0; ch < nchunks; ++ch) {
+            const int64_t j1 = (ch + 1) * chunk < P ? (ch + 1) * chunk : P;
+            orc_local_step(n, P, ch * chunk, j1, x, v, h, c, noise_bf16, seed, k, gamma, mu, wd, sigma);
+        }
+        if (!sync_now(s, st, k)) continue;
+        #pragma omp parallel for num_threads(threads) schedule(static)
+        for (int64_t ch = 0; ch < nchunks; ++ch) {
+            const int64_t j1 = (ch + 1) * chunk < P ? (ch + 1) * chunk : P;
+            partD[ch] = 0.0;
+            partL[ch] = 0.0;
+            orc_average_variance(n, P, ch * chunk, j1, x, h, c, &partD[ch], &partL[ch]);
+        }
+        double D = 0.0, loss = 0.0;
+        for (int64_t ch = 0; ch < nchunks; ++ch) {
+            D += partD[ch];
+            loss += partL[ch];
+        }
+        double S = D / (double)n;
+        int32_t phase = orc_on_sync(s, st, k, S, (double)gamma);
+        if (tr != NULL && syncs < tr->cap) {
+            tr->k[syncs] = k;
+            tr->p[syncs] = st->p;
+            tr->S[syncs] = S;
+            tr->C2[syncs] = st->C2;
+            tr->loss[syncs] = loss;
+            tr->phase[syncs] = phase;
+        }
+        syncs = syncs + 1;
+    }
+    free(part);
     return syncs;
 }
 

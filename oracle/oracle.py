@@ -4,7 +4,8 @@ TEST INFRASTRUCTURE ONLY: the tests, ``__graft_entry__.smoke()`` and the CPU
 baseline leg of ``bench.py`` may use this module; the product path never does.
 It shares no code with the CUDA library: it compiles its own C file with gcc
 (``-O2 -ffp-contract=off``, no fast-math, so every fp32 operation is one IEEE
-rounding) and marshals numpy arrays through ctypes.
+rounding; ``-fopenmp`` for the chunked all-core run) and marshals numpy arrays
+through ctypes.
 
 Every function cites the part of the paper it follows (Jiang & Agrawal,
 "Adaptive Periodic Averaging", arXiv 2007.06134); the C file states the
@@ -26,8 +27,9 @@ _LIB = os.path.join(_HERE, "liboracle_adpsgd.so")
 _lock = threading.Lock()
 _lib = None
 
-CFLAGS = ["-O2", "-std=c11", "-fPIC", "-shared", "-ffp-contract=off", "-fno-fast-math",
+CFLAGS = ["-O2", "-std=c11", "-fPIC", "-shared", "-fopenmp", "-ffp-contract=off", "-fno-fast-math",
           "-fno-unsafe-math-optimizations"]
+CHUNK_COLUMNS = 1 << 16  # columns per chunk of the all-core run
 
 
 def build(force: bool = False) -> str:
@@ -134,6 +136,8 @@ def lib():
                                   C.POINTER(Schedule), C.POINTER(State), C.c_int64, C.c_int64,
                                   C.POINTER(Trace)]
             L.orc_run.restype = C.c_int64
+            L.orc_run_chunked.argtypes = [C.c_int32, C.c_int64] + L.orc_run.argtypes
+            L.orc_run_chunked.restype = C.c_int64
             L.orc_schedule_only.argtypes = [C.POINTER(Schedule), C.POINTER(C.c_double), C.c_int64,
                                             C.POINTER(C.c_int64), C.POINTER(C.c_int32), C.c_int64]
             L.orc_schedule_only.restype = C.c_int64
@@ -318,10 +322,22 @@ class RunTrace:
     var: np.ndarray = None
 
 
+def host_threads() -> int:
+    """Host cores this process may run on."""
+    try:
+        return len(os.sched_getaffinity(0))
+    except AttributeError:  # pragma: no cover - Linux has sched_getaffinity
+        return os.cpu_count() or 1
+
+
 def run(x, v, h, c, *, spec: ScheduleSpec, seed, mu, wd, sigma, noise=None, state=None,
-        k_begin=0, k_end=None, cap=100000, track_variance=False) -> RunTrace:
+        k_begin=0, k_end=None, cap=100000, track_variance=False, threads=None,
+        chunk=CHUNK_COLUMNS) -> RunTrace:
     """Algorithm 2 (or 1) end to end on the [n, P] arrays, in place; returns the sync trace and,
-    with track_variance, Var[W_k] at the start of every iteration k (Sec. III, Eq. vt)."""
+    with track_variance, Var[W_k] at the start of every iteration k (Sec. III, Eq. vt).
+    threads=None runs on one thread in column order; threads=t (e.g. host_threads()) runs the
+    chunked all-core form: the same x, v and schedule, D and the loss summed per chunk of `chunk`
+    columns in chunk order."""
     _check_state(x, v)
     n, P = x.shape
     k_end = spec.K if k_end is None else k_end
@@ -336,8 +352,14 @@ def run(x, v, h, c, *, spec: ScheduleSpec, seed, mu, wd, sigma, noise=None, stat
     h = np.ascontiguousarray(h, dtype=np.float32)
     c = np.ascontiguousarray(c, dtype=np.float32)
     nz = None if noise is None else _u16p(np.ascontiguousarray(noise, dtype=np.uint16))
-    syncs = lib().orc_run(n, P, _f32p(x), _f32p(v), _f32p(h), _f32p(c), nz, seed, mu, wd, sigma,
-                          C.byref(s), C.byref(st), k_begin, k_end, C.byref(tr))
+    args = (n, P, _f32p(x), _f32p(v), _f32p(h), _f32p(c), nz, seed, mu, wd, sigma,
+            C.byref(s), C.byref(st), k_begin, k_end, C.byref(tr))
+    if threads is None:
+        syncs = lib().orc_run(*args)
+    else:
+        syncs = lib().orc_run_chunked(threads, chunk, *args)
+        if syncs < 0:
+            raise ValueError(f"chunked run refused: chunk {chunk} must be a positive multiple of 4")
     m = min(syncs, cap)
     return RunTrace(**{a: b[:m].copy() for a, b in arrs.items()}, syncs=syncs, var=var)
 
