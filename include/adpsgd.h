@@ -213,11 +213,16 @@ int adpsgd_average_and_variance(adpsgd_ctx* ctx, double* D_out, double* loss_out
  * stream: cudaStream_t as void*.  wait_timeout_ms bounds the wait for the stream (<= 0: 60000).
  *
  * The first call on each device looks up the scratch array's device address
- * (cudaGetSymbolAddress).  Make that first call before any stream capture.  Every call uses the
- * same array, which keeps the last call's contents.  Each call clears the completion counter in
- * it on the stream before the launch, and writes every other slot before reading it.  Calls that
- * overlap on the GPU (several host threads, or streams that run concurrently) race on the array
- * and must be serialised by the caller.
+ * (cudaGetSymbolAddress) with that device current.  Make that first call before any stream
+ * capture.  The address is cached with the id of the CUDA context it was looked up in; a call from
+ * a different context (after cudaDeviceReset, or with another context current) looks it up again.
+ * Every call uses the same array, which keeps the last call's contents.  Each call clears the
+ * completion counter in it on the stream before the launch, and writes every other slot before
+ * reading it.  Calls that overlap on the GPU (several host threads, or streams that run
+ * concurrently) race on the array and must be serialised by the caller.
+ * The call returns once the stream has passed the averaging (a bounded poll, then a 16-byte copy
+ * of the two sums).  After ADPSGD_E_TIMEOUT the averaging may still be running on the shared
+ * array: wait for that stream to finish before calling again, on any stream.
  * Errors: E_INVAL, E_ALIGN, E_TIMEOUT, E_CUDA. */
 int adpsgd_average_and_variance_static(float* x, const float* h, const float* c, int32_t n, int64_t P,
                                        double* D_out, double* loss_out, int64_t wait_timeout_ms, void* stream);
@@ -290,8 +295,10 @@ int adpsgd_noise_fill_bf16(uint64_t seed, int32_t n, int64_t P, uint16_t* out, v
  * host buffer is page-locked (cudaHostAlloc, cudaHostRegister, PyTorch pinned memory), the
  * library's copy kernel moves the bytes through the buffer's mapped device address.  That
  * holds its throughput when other work loads the host memory, where the copy engines slow
- * down.  Any other host memory goes through cudaMemcpyAsync.  The device side must be device
- * (or managed) memory.  Both pointers 16-byte aligned; bytes need not be a multiple of 16.
+ * down.  The kernel is used only when the device side is device memory of the current device;
+ * managed memory, another device's memory, and host memory that is not page-locked go through
+ * cudaMemcpyAsync.  The device side must be device (or managed) memory.  Both pointers 16-byte
+ * aligned; bytes need not be a multiple of 16.
  * bytes == 0 does nothing.  The caller keeps both buffers alive until the stream has passed
  * the copy.
  * Errors: E_INVAL (NULL pointer with bytes > 0, bytes < 0, the device side not device memory,

@@ -21,6 +21,7 @@
 // Every fp32 operation of the update, the mean and the generator is written out once and
 // compiled with -fmad=false, so results are bit-identical to any IEEE evaluation of the same
 // sequence.
+#include <cuda.h>
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 
@@ -398,15 +399,47 @@ static __device__ __align__(256) double g_static_scratch[2 * adpsgd::kStaticMaxB
 namespace adpsgd {
 
 namespace {
+
 std::mutex g_static_mutex;
-double* g_static_address[kStaticMaxDevices] = {};
+
+// The address of g_static_scratch as seen by one CUDA context.  A module's globals move when its
+// context is destroyed and created again (cudaDeviceReset, a primary-context reset, or another
+// context made current), so the cached address is tied to the context's process-unique id.
+struct StaticAddress {
+    unsigned long long context_id = 0;
+    double* address = nullptr;
+};
+StaticAddress g_static_address[kStaticMaxDevices];
+
+using CtxGetIdFn = CUresult (*)(CUcontext, unsigned long long*);
+
+// Id of the current context (cuCtxGetId with a null context), found through the runtime's
+// driver entry-point lookup so that the library needs no link against the driver library.
+cudaError_t current_context_id(unsigned long long* id)
+{
+    static CtxGetIdFn get_id = nullptr;
+    static bool looked_up = false;
+    if (!looked_up) {
+        void* fn = nullptr;
+        cudaDriverEntryPointQueryResult found = cudaDriverEntryPointSymbolNotFound;
+        const cudaError_t e = cudaGetDriverEntryPointByVersion("cuCtxGetId", &fn, 12000, cudaEnableDefault, &found);
+        if (e != cudaSuccess) return e;
+        if (found != cudaDriverEntryPointSuccess || fn == nullptr) return cudaErrorSymbolNotFound;
+        get_id = reinterpret_cast<CtxGetIdFn>(fn);
+        looked_up = true;
+    }
+    return get_id(nullptr, id) == CUDA_SUCCESS ? cudaSuccess : cudaErrorDeviceUninitialized;
+}
+
 }  // namespace
 
 int static_scratch_max_blocks() { return kStaticMaxBlocks; }
 
-// Device address of g_static_scratch on the current device.  On host, the symbol's name is
-// only a stand-in, not a device address, so it is looked up once per device (with that device
-// current) and cached.
+// Device address of g_static_scratch in the current device's current context.  In host code the
+// symbol's name is only a stand-in, not a device address, so the address is looked up with
+// cudaGetSymbolAddress (with that device current) the first time a context calls, and cached
+// with the context's id.  cudaGetSymbolAddress also creates the runtime's context if there is
+// none yet, so the id is read after it on a first call.
 cudaError_t static_scratch_address(double** partials, double** out, unsigned int** counter)
 {
     int device = 0;
@@ -414,15 +447,21 @@ cudaError_t static_scratch_address(double** partials, double** out, unsigned int
     if (e != cudaSuccess) return e;
     if (device < 0 || device >= kStaticMaxDevices) return cudaErrorInvalidDevice;
     std::lock_guard<std::mutex> lock(g_static_mutex);
-    if (g_static_address[device] == nullptr) {
+    StaticAddress& slot = g_static_address[device];
+    unsigned long long id = 0;
+    const bool have_id = current_context_id(&id) == cudaSuccess;
+    if (!have_id || slot.address == nullptr || slot.context_id != id) {
         void* address = nullptr;
         e = cudaGetSymbolAddress(&address, g_static_scratch);
         if (e != cudaSuccess) return e;
-        g_static_address[device] = static_cast<double*>(address);
+        e = current_context_id(&id);
+        if (e != cudaSuccess) return e;
+        slot.context_id = id;
+        slot.address = static_cast<double*>(address);
     }
-    *partials = g_static_address[device];
-    *out = g_static_address[device] + 2 * kStaticMaxBlocks;
-    *counter = reinterpret_cast<unsigned int*>(g_static_address[device] + 2 * kStaticMaxBlocks + 2);
+    *partials = slot.address;
+    *out = slot.address + 2 * kStaticMaxBlocks;
+    *counter = reinterpret_cast<unsigned int*>(slot.address + 2 * kStaticMaxBlocks + 2);
     return cudaSuccess;
 }
 

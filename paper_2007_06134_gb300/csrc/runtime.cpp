@@ -824,13 +824,15 @@ int adpsgd_noise_fill_bf16(uint64_t seed, int32_t n, int64_t P, uint16_t* out, v
 
 namespace {
 
-// The kind of memory p points into (cudaMemoryTypeUnregistered for plain host memory).
-cudaError_t memory_type(const void* p, cudaMemoryType* type)
+// The kind of memory p points into (cudaMemoryTypeUnregistered for plain host memory) and,
+// for device memory, the device it lives on.
+cudaError_t memory_type(const void* p, cudaMemoryType* type, int* device)
 {
     cudaPointerAttributes attr;
     const cudaError_t e = cudaPointerGetAttributes(&attr, p);
     if (e != cudaSuccess) return e;
     *type = attr.type;
+    *device = attr.device;
     return cudaSuccess;
 }
 
@@ -844,8 +846,9 @@ int transfer(void* dst, const void* src, int64_t bytes, void* stream, bool to_de
     const void* host = to_device ? src : dst;
     const void* device = to_device ? dst : src;
     cudaMemoryType host_type, device_type;
-    cudaError_t e = memory_type(device, &device_type);
-    if (e == cudaSuccess) e = memory_type(host, &host_type);
+    int host_dev = -1, device_dev = -1, current = 0;
+    cudaError_t e = memory_type(device, &device_type, &device_dev);
+    if (e == cudaSuccess) e = memory_type(host, &host_type, &host_dev);
     if (e != cudaSuccess) return cuda_fail(e, "cudaPointerGetAttributes");
     if (device_type != cudaMemoryTypeDevice && device_type != cudaMemoryTypeManaged) {
         g_last_error = "the device side of the copy is not device memory";
@@ -855,13 +858,20 @@ int transfer(void* dst, const void* src, int64_t bytes, void* stream, bool to_de
         g_last_error = "the host side of the copy is device memory";
         return ADPSGD_E_INVAL;
     }
+    e = cudaGetDevice(&current);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     void* mapped = nullptr;
-    if (host_type == cudaMemoryTypeHost && cudaHostGetDevicePointer(&mapped, const_cast<void*>(host), 0) == cudaSuccess &&
-        aligned16(mapped)) {
-        int device_id = 0, sms = 0;
-        e = cudaGetDevice(&device_id);
-        if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, device_id);
+    // The copy kernel runs on the current device, so it takes only device memory of that device;
+    // managed memory and another device's memory go through cudaMemcpyAsync, which needs no peer
+    // mapping and migrates managed pages itself.
+    const bool kernel_route = device_type == cudaMemoryTypeDevice && device_dev == current &&
+                              host_type == cudaMemoryTypeHost &&
+                              cudaHostGetDevicePointer(&mapped, const_cast<void*>(host), 0) == cudaSuccess &&
+                              aligned16(mapped);
+    if (kernel_route) {
+        int sms = 0;
+        e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, current);
         if (e != cudaSuccess) return cuda_fail(e, "device query");
         e = to_device ? adpsgd::launch_copy(dst, mapped, bytes, sms, s) : adpsgd::launch_copy(mapped, src, bytes, sms, s);
         return e == cudaSuccess ? ADPSGD_OK : cuda_fail(e, "copy kernel");

@@ -5,6 +5,10 @@ cudaMemcpyAsync.  Both must deliver every byte, including ragged tails, interior
 pinned allocation, and empty copies.  Bad arguments are refused before anything is enqueued.
 A whole run fed and read back through these calls matches the oracle.
 """
+import ctypes as C
+import os
+import subprocess
+
 import numpy as np
 import pytest
 
@@ -63,6 +67,42 @@ def test_copies_are_stream_ordered():
         abi.adpsgd_copy_d2h(out, dev, stream=s)
     s.synchronize()
     assert torch.equal(out, 2.0 * src)
+
+
+@pytest.fixture(scope="module")
+def managed(tmp_path_factory):
+    src = os.path.join(os.path.dirname(__file__), "cuda", "managed_alloc.cu")
+    so = str(tmp_path_factory.mktemp("managed") / "libmanaged_alloc.so")
+    subprocess.check_call(["nvcc", "-gencode", "arch=compute_103a,code=sm_103a", "-O2", "-shared",
+                           "-Xcompiler", "-fPIC", "-o", so, src])
+    lib = C.CDLL(so)
+    lib.test_alloc_managed.argtypes = [C.c_size_t]
+    lib.test_alloc_managed.restype = C.c_void_p
+    lib.test_free_managed.argtypes = [C.c_void_p]
+    lib.test_free_managed.restype = C.c_int
+    return lib
+
+
+@pytest.mark.parametrize("nbytes", [16, 4096 + 3, (8 << 20) + 5])
+def test_managed_device_side(managed, nbytes):
+    # The copy kernel takes only device memory of the current device; a managed buffer goes
+    # through cudaMemcpyAsync and must still receive and return every byte.
+    torch.cuda.synchronize()
+    ptr = managed.test_alloc_managed(nbytes + 16)
+    assert ptr
+    try:
+        src = _bytes(nbytes, 7 + nbytes, True)
+        abi.adpsgd_copy_h2d(ptr, src, nbytes)
+        torch.cuda.synchronize()
+        got = np.ctypeslib.as_array((C.c_uint8 * nbytes).from_address(ptr)).copy()
+        assert np.array_equal(got, src.numpy())
+        back = torch.zeros(nbytes, dtype=torch.uint8).pin_memory()
+        abi.adpsgd_copy_d2h(back, ptr, nbytes)
+        torch.cuda.synchronize()
+        assert torch.equal(back, src)
+    finally:
+        torch.cuda.synchronize()
+        assert managed.test_free_managed(ptr) == 0
 
 
 def test_bad_arguments_are_refused():

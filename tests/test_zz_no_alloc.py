@@ -71,3 +71,37 @@ def test_static_scratch_entry_without_loss_and_argument_checks():
     with pytest.raises(abi.AdpsgdError) as e:
         abi.adpsgd_average_and_variance_static(xd, None, None, 0, P, want_loss=False)
     assert e.value.status == abi.E_INVAL
+
+
+def test_static_scratch_entry_refuses_misaligned_x():
+    n, P = 2, 4096
+    xd = torch.zeros(n * P + 4, device=DEV)
+    with pytest.raises(abi.AdpsgdError) as e:
+        abi.adpsgd_average_and_variance_static(xd[1:], None, None, n, P, want_loss=False)
+    assert e.value.status == abi.E_ALIGN
+
+
+def test_static_scratch_entry_bounded_wait_behind_queued_work():
+    # A short wait limit behind work already queued on the stream returns E_TIMEOUT without
+    # blocking; once the stream has drained, the next call returns the right sums.
+    w = inputs.WORKLOADS["resnet18-n8"]
+    n, P = 8, 1 << 22
+    h, c = inputs.problem(w, P)
+    busy_x = torch.zeros((n, P), device=DEV)
+    busy_v = torch.zeros_like(busy_x)
+    x, _ = inputs.random_state(4, 4096, 21)
+    ref_x, ref_D, _ = _with_context(x, np.ones(4096, np.float32), np.zeros(4096, np.float32))
+    xd = _dev(x)
+    with abi.adpsgd_init(abi.make_config(n, P), busy_x, busy_v, _dev(h), _dev(c)) as ctx:
+        abi.adpsgd_local_steps(ctx, 0, [0.01] * 400)  # tens of milliseconds of queued work
+        with pytest.raises(abi.AdpsgdError) as e:
+            abi.adpsgd_average_and_variance_static(xd, None, None, 4, 4096, want_loss=False, wait_timeout_ms=1)
+        assert e.value.status == abi.E_TIMEOUT
+        torch.cuda.synchronize()
+    assert np.array_equal(xd.cpu().numpy(), ref_x)  # the timed-out averaging still ran to the end
+    D, _ = abi.adpsgd_average_and_variance_static(xd, None, None, 4, 4096, want_loss=False)
+    assert D == 0.0  # averaged replicas have no spread
+    xd.copy_(_dev(x))
+    D, _ = abi.adpsgd_average_and_variance_static(xd, None, None, 4, 4096, want_loss=False)
+    torch.cuda.synchronize()
+    assert _rel(D, ref_D) <= REL
