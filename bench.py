@@ -1,13 +1,14 @@
 #!/usr/bin/env python3
 """Benchmark of the ADPSGD hot path on GB300: one JSON line on stdout.
 
-A step is one whole ADPSGD run of the resnet18-n8 workload (n = 8 replicas of a
-ResNet-18-sized fp32 vector, P = 11,689,512; 2000 iterations; step size 0.1, x0.1 at
-iterations 1000 and 1500; momentum 0.9, weight decay 5e-4, noise sigma 1; Algorithm 2 with
-p_init = 4 and K_s = 500): every iteration one fused local-step launch over all replicas,
-every sync one fused average + variance launch, the period rule on the host.  Inputs are
-resident in HBM when the timed region starts (x and v are reset to x0 = 0 inside it);
-x and v (748 MB) are larger than L2, so no flush is needed between steps.
+A step is one whole ADPSGD run of the vgg16-n8 workload (n = 8 replicas of a VGG-16-sized fp32
+vector, P = 138,357,544; 500 iterations; step size 0.05; momentum 0.9, weight decay 5e-4, noise
+sigma 0.5; curvatures LogUniform[1e-3, 1], minimisers N(0, 0.1^2); Algorithm 2 with p_init = 4
+and K_s = 125): every iteration one fused local-step launch over all replicas, every sync one
+launch that fuses that iteration's step with the average + variance, the period rule on the
+host.  Inputs are resident in HBM when the timed region starts (x and v are reset to x0 = 0
+inside it); x and v (8.9 GB) are far larger than L2, so no flush is needed between steps.
+Other workloads: --workload resnet18-n8, resnet50-n16-bf16noise, quadratic-n4-P1M.
 
 value      replica-params/s of the whole run (n * P * iterations / step time), all ranks
 e2e        the same through the C ABI with host buffers: H2D of x0, v0, h, c and D2H of the
@@ -15,12 +16,14 @@ e2e        the same through the C ABI with host buffers: H2D of x0, v0, h, c and
 roofline   the local-step kernel (the dominant one): algorithmic bytes per launch
            (16 n P + 8 P) over its mean CUDA-event duration (events around every 4th launch in
            the timed region), against the measured HBM copy bandwidth; avg_variance reports
-           the averaging kernel the same way (8 n P + 8 P)
-cpu_baseline  the CPU oracle on a bounded sample of the same workload, one host core
+           the averaging kernel the same way (8 n P + 8 P), sync_step the fused sync step
+cpu_baseline  the CPU oracle on a bounded sample of the same workload: on every host core
+           (the chunked run) and on one core
 
---impl reference times the CPU oracle itself (the only reference this build has) on bounded
-samples of the same workload.  Under torchrun every rank runs its own independent problem
-(weak scaling; the path has no cross-rank exchange) and rank 0 prints the max-over-ranks time.
+--impl reference times the CPU oracle itself (the only reference this build has) on every host
+core, on bounded samples of the same workload.  Under torchrun (N ranks, one GPU each) the one
+problem is split by columns: each rank holds its column range of x, v, h and c, and the ranks
+exchange two fp64 partial sums per sync (strong scaling); rank 0 prints the max-over-ranks time.
 """
 from __future__ import annotations
 
@@ -39,10 +42,16 @@ sys.path.insert(0, ROOT)
 
 METRIC = "avg+variance GB/s vs HBM peak; fused local-step replica-params/sec"
 UNIT = "replica-params/s"
-CPU_SAMPLE_COLUMNS = 1 << 20
+DEFAULT_WORKLOAD = "vgg16-n8"
 TIMING_PERIOD = 4  # kernel durations from CUDA events around every 4th launch of each kernel
 AVG_SAMPLES = 24  # timed standalone averaging launches
+# Bounded oracle samples: the workload's first columns, all replicas, a few iterations with a
+# sync every 4 (one core: 2^21 columns; every core: 2^24 columns), a few seconds each.
 CPU_SAMPLE_ITERS = 24
+CPU_SAMPLE_COLUMNS_ONE_CORE = 1 << 21
+CPU_SAMPLE_COLUMNS_ALL_CORES = 1 << 24
+# The workload whose ncu capture gives DRAM bytes per replica-param for the others.
+TRAFFIC_CAPTURE_WORKLOAD = "resnet18-n8"
 
 
 def log(*a):
@@ -85,17 +94,27 @@ def kernel_source_digest(kernel: str) -> str:
     return h.hexdigest()[:16]
 
 
-def recorded_traffic(kernel: str, workload: str):
-    """DRAM bytes per launch from a committed ncu capture, if the kernel source is unchanged since."""
+def recorded_traffic(kernel: str, workload: str, algorithmic_bytes: int):
+    """DRAM bytes per launch from a committed ncu capture, if the kernel source is unchanged since:
+    (bytes, how).  A workload without its own capture takes the capture of
+    TRAFFIC_CAPTURE_WORKLOAD scaled by the ratio of algorithmic bytes per launch (the kernels
+    stream their arrays once, so traffic grows in proportion to the replica-params processed)."""
     path = os.path.join(ROOT, "profiles", "traffic.json")
     if not os.path.exists(path):
-        return None
+        return None, None
     with open(path) as f:
         d = json.load(f)
-    e = d.get(kernel, {}).get(workload)
+    rows = d.get(kernel, {})
+    e = rows.get(workload)
+    how = "ncu capture of this workload"
+    scale = 1.0
+    if e is None and TRAFFIC_CAPTURE_WORKLOAD in rows:
+        e = rows[TRAFFIC_CAPTURE_WORKLOAD]
+        scale = algorithmic_bytes / e["algorithmic_bytes_per_launch"]
+        how = f"ncu capture of {TRAFFIC_CAPTURE_WORKLOAD} scaled by algorithmic bytes ({scale:.4f})"
     if not e or e.get("source_sha256_16") != kernel_source_digest(kernel):
-        return None
-    return e["dram_bytes_per_launch"]
+        return None, None
+    return int(round(e["dram_bytes_per_launch"] * scale)), how
 
 
 # ------------------------------------------------------------------------------------------
@@ -158,7 +177,7 @@ class ClockSampler:
 
 
 # ------------------------------------------------------------------------------------------
-# distributed plumbing (barrier + max over ranks only; no data-path collective)
+# distributed plumbing (barrier, max over ranks; the per-sync exchange is shard.dist_gather)
 # ------------------------------------------------------------------------------------------
 
 def dist_setup(args):
@@ -198,12 +217,34 @@ def barrier(pg, device=None):
 # CPU oracle leg
 # ------------------------------------------------------------------------------------------
 
-def oracle_sample(w, seed_offset=0):
+def cpu_model() -> str:
+    """The host CPU's model name (x86: /proc/cpuinfo; Arm: lscpu), or the machine type."""
+    try:
+        with open("/proc/cpuinfo") as f:
+            for line in f:
+                if line.lower().startswith("model name"):
+                    return line.split(":", 1)[1].strip()
+    except OSError:
+        pass
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for line in out.splitlines():
+            if line.strip().lower().startswith("model name"):
+                return line.split(":", 1)[1].strip()
+    except Exception:
+        pass
+    import platform
+    return platform.machine()
+
+
+def oracle_sample(w, seed_offset=0, threads=None):
     """Time the oracle on a bounded sample: CPU_SAMPLE_ITERS iterations of the workload's local step
-    and its syncs (constant period 4) on its first CPU_SAMPLE_COLUMNS columns, all replicas."""
+    and its syncs (constant period 4) on its first columns, all replicas.  threads=None: the
+    single-thread run on CPU_SAMPLE_COLUMNS_ONE_CORE columns; threads=t: the chunked run on t host
+    threads on CPU_SAMPLE_COLUMNS_ALL_CORES columns.  Returns (replica-params/s, seconds, text)."""
     from oracle import oracle as O
     from paper_2007_06134_gb300 import inputs
-    P = min(CPU_SAMPLE_COLUMNS, w.P)
+    P = min(CPU_SAMPLE_COLUMNS_ONE_CORE if threads is None else CPU_SAMPLE_COLUMNS_ALL_CORES, w.P)
     h, c = inputs.problem(w, P)
     x, v = inputs.zero_state(w.n, P)
     noise = O.noise_bf16(w.seed, w.n, P) if w.noise == "bf16" else None
@@ -211,32 +252,48 @@ def oracle_sample(w, seed_offset=0):
                           milestones=w.milestones)
     O.build()
     t0 = time.perf_counter()
-    O.run(x, v, h, c, spec=spec, seed=w.seed + seed_offset, mu=w.mu, wd=w.wd, sigma=w.sigma, noise=noise)
+    O.run(x, v, h, c, spec=spec, seed=w.seed + seed_offset, mu=w.mu, wd=w.wd, sigma=w.sigma, noise=noise,
+          threads=threads)
     dt = time.perf_counter() - t0
     rp = w.n * P * CPU_SAMPLE_ITERS
+    how = "one core" if threads is None else f"{threads} host threads (chunked run)"
     return rp / dt, dt, (f"{CPU_SAMPLE_ITERS} iterations (syncs every 4) of {w.name} on its first {P} columns, "
-                         f"all {w.n} replicas: {rp} replica-param updates in {dt:.2f} s")
+                         f"all {w.n} replicas, {how}: {rp} replica-param updates in {dt:.2f} s")
+
+
+def cpu_baseline(w):
+    """The oracle on every host core (the reported figure) and on one core."""
+    from oracle import oracle as O
+    threads = O.host_threads()
+    r_all, _, sample_all = oracle_sample(w, threads=threads)
+    r_one, _, sample_one = oracle_sample(w)
+    return {"value": r_all, "unit": UNIT, "cores": threads, "kind": "oracle", "sample": sample_all,
+            "cpu_model": cpu_model(),
+            "single_core": {"value": r_one, "unit": UNIT, "cores": 1, "sample": sample_one}}
 
 
 def run_reference(args, w):
     world, rank, local, pg = dist_setup(args)
     if rank != 0:
         return 0
+    from oracle import oracle as O
+    threads = O.host_threads()
     for _ in range(args.warmup):
-        oracle_sample(w)
+        oracle_sample(w, threads=threads)
     rates, times, sample = [], [], ""
     for s in range(args.steps):
-        r, dt, sample = oracle_sample(w, s + 1)
+        r, dt, sample = oracle_sample(w, s + 1, threads=threads)
         rates.append(r)
         times.append(dt)
     value = float(np.mean(rates))
     line = {
         "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1000.0 * float(np.mean(times)),
-        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
-        "config": {"workload": w.name, "n": w.n, "P": w.P, "K": w.K, "sample_columns": min(CPU_SAMPLE_COLUMNS, w.P),
-                   "sample_iterations": CPU_SAMPLE_ITERS},
-        "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": sample},
+        "higher_is_better": True, "scaling": "strong", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+        "config": {"workload": w.name, "n": w.n, "P": w.P, "K": w.K,
+                   "sample_columns": min(CPU_SAMPLE_COLUMNS_ALL_CORES, w.P), "sample_iterations": CPU_SAMPLE_ITERS},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": threads, "kind": "oracle", "sample": sample,
+                         "cpu_model": cpu_model()},
         "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
     print(json.dumps(line), flush=True)
@@ -255,17 +312,22 @@ def schedule_for(abi, w):
 def run_gpu(args, w):
     import torch
 
-    from paper_2007_06134_gb300 import abi, inputs
+    from paper_2007_06134_gb300 import abi, inputs, shard
 
     world, rank, local, pg = dist_setup(args)
     device = torch.device("cuda", local)
     torch.cuda.set_device(device)
     stream = torch.cuda.current_stream(device)
     abi.load()
-    seed = w.seed + rank  # independent problem per rank
+    seed = w.seed
 
-    h, c = inputs.problem(w)
-    n, P = w.n, w.P
+    # One problem; with N ranks each rank holds a contiguous column range of it (strong scaling).
+    n, P_total = w.n, w.P
+    col0, P = shard.column_split(P_total, world, rank)
+    gather = shard.dist_gather()[0] if world > 1 else None
+    h_all, c_all = inputs.problem(w)
+    h, c = np.ascontiguousarray(h_all[col0:col0 + P]), np.ascontiguousarray(c_all[col0:col0 + P])
+    del h_all, c_all
     hd = torch.from_numpy(h).to(device)
     cd = torch.from_numpy(c).to(device)
     xd = torch.zeros((n, P), dtype=torch.float32, device=device)
@@ -273,13 +335,20 @@ def run_gpu(args, w):
     noise = None
     if w.noise == "bf16":
         noise = torch.empty((n, P), dtype=torch.int16, device=device)
-        abi.adpsgd_noise_fill_bf16(w.seed, n, P, noise, stream)
+        abi.adpsgd_noise_fill_bf16_shard(w.seed, n, P, col0, noise, stream)
     fuse_sync = not args.no_sync_fusion
-    cfg = abi.make_config(n, P, momentum=w.mu, weight_decay=w.wd, noise_sigma=w.sigma, seed=seed,
-                          noise_mode=abi.NOISE_BF16 if noise is not None else abi.NOISE_PHILOX, want_loss=True,
-                          time_kernels=TIMING_PERIOD, fuse_sync_step=fuse_sync)
+    noise_mode = abi.NOISE_BF16 if noise is not None else abi.NOISE_PHILOX
+
+    def context(exchange=True, **kw):
+        cfg = abi.make_config(n, P, momentum=w.mu, weight_decay=w.wd, noise_sigma=w.sigma, seed=seed,
+                              noise_mode=noise_mode, want_loss=True, **kw)
+        ctx = abi.adpsgd_init(cfg, xd, vd, hd, cd, noise, stream)
+        if world > 1 and exchange:
+            abi.adpsgd_set_shard(ctx, abi.make_shard(world, rank, col0, P_total, gather))
+        return ctx
+
     sched = schedule_for(abi, w)
-    ctx = abi.adpsgd_init(cfg, xd, vd, hd, cd, noise, stream)
+    ctx = context(time_kernels=TIMING_PERIOD, fuse_sync_step=fuse_sync)
 
     def one_run():
         xd.zero_()
@@ -316,8 +385,9 @@ def run_gpu(args, w):
     ms_total = ev0.elapsed_time(ev1)
     ms_total = max_over_ranks(pg, ms_total, device)
     ms_step = ms_total / args.steps
-    rp_per_step = n * P * w.K
-    value = world * rp_per_step / (ms_step / 1000.0)
+    rp_per_step = n * P_total * w.K  # the whole problem, all ranks together
+    value = rp_per_step / (ms_step / 1000.0)
+    launches = int(max_over_ranks(pg, float(launches), device)) * world
 
     kt = abi.adpsgd_kernel_times(ctx)
     kt = dict(kt)
@@ -331,11 +401,10 @@ def run_gpu(args, w):
     clock_summary = clocks.summary()
 
     # The averaging kernel on its own, as the unfused path runs it: one launch after each local
-    # step, every launch timed (with fused sync steps the run above launches few of them).
+    # step, every launch timed (with fused sync steps the run above launches few of them).  Only
+    # the kernel is timed here, so this context does not exchange its sums.
     k2_bytes = 8 * n * P + 8 * P
-    cfg_k2 = abi.make_config(n, P, momentum=w.mu, weight_decay=w.wd, noise_sigma=w.sigma, seed=seed,
-                             noise_mode=cfg.noise_mode, want_loss=True, time_kernels=1)
-    with abi.adpsgd_init(cfg_k2, xd, vd, hd, cd, noise, stream) as ctx_k2:
+    with context(exchange=False, time_kernels=1) as ctx_k2:
         for r in range(AVG_SAMPLES + 2):
             if r == 2:
                 abi.adpsgd_reset_kernel_times(ctx_k2)
@@ -353,11 +422,9 @@ def run_gpu(args, w):
         hh = torch.from_numpy(h).pin_memory()
         ch = torch.from_numpy(c).pin_memory()
         xout = torch.empty_like(x0h).pin_memory()
-        h2d = 4 * (2 * n * P + 2 * P)
-        d2h = 4 * n * P
-        cfg_e2e = abi.make_config(n, P, momentum=w.mu, weight_decay=w.wd, noise_sigma=w.sigma, seed=seed,
-                                  noise_mode=cfg.noise_mode, want_loss=True, fuse_sync_step=fuse_sync)
-        ctx_e2e = abi.adpsgd_init(cfg_e2e, xd, vd, hd, cd, noise, stream)  # set-up, outside the timed region
+        h2d = 4 * (2 * n * P_total + 2 * P_total)  # all ranks together
+        d2h = 4 * n * P_total
+        ctx_e2e = context(fuse_sync_step=fuse_sync)  # set-up, outside the timed region
 
         marks = [torch.cuda.Event(enable_timing=True) for _ in range(4)]
 
@@ -383,7 +450,7 @@ def run_gpu(args, w):
         log("e2e last step: h2d %.1f ms, run %.1f ms, d2h %.1f ms" % (
             marks[0].elapsed_time(marks[1]), marks[1].elapsed_time(marks[2]), marks[2].elapsed_time(marks[3])))
         dt = max_over_ranks(pg, (time.perf_counter() - t0) / e2e_steps, device)
-        e2e_value = world * rp_per_step / dt
+        e2e_value = rp_per_step / dt
         e2e_phases = {"h2d_ms": marks[0].elapsed_time(marks[1]), "run_ms": marks[1].elapsed_time(marks[2]),
                       "d2h_ms": marks[2].elapsed_time(marks[3]), "wall_ms": dt * 1000.0}
         ctx_e2e.close()
@@ -391,10 +458,7 @@ def run_gpu(args, w):
     # The same run with each sync interval fused into one kernel (separable objective only).
     fused = None
     if not args.no_fused and n <= 32:
-        cfg_f = abi.make_config(n, P, momentum=w.mu, weight_decay=w.wd, noise_sigma=w.sigma, seed=seed,
-                                noise_mode=cfg.noise_mode, want_loss=True, time_kernels=TIMING_PERIOD,
-                                fuse_intervals=True)
-        with abi.adpsgd_init(cfg_f, xd, vd, hd, cd, noise, stream) as ctx_f:
+        with context(time_kernels=TIMING_PERIOD, fuse_intervals=True) as ctx_f:
             def fused_run():
                 xd.zero_()
                 vd.zero_()
@@ -410,7 +474,7 @@ def run_gpu(args, w):
             torch.cuda.synchronize(device)
             fms = max_over_ranks(pg, ev0.elapsed_time(ev1), device) / args.steps
             ft = abi.adpsgd_kernel_times(ctx_f)
-        fused = {"value": world * rp_per_step / (fms / 1000.0), "unit": UNIT, "ms_per_step": fms,
+        fused = {"value": rp_per_step / (fms / 1000.0), "unit": UNIT, "ms_per_step": fms,
                  "interval_launches_per_step": fstats.interval_launches,
                  "interval_ms_per_launch": ft["interval_ms"] / max(1, ft["interval_launches"]),
                  "note": "each sync interval (local steps + averaging) as one kernel; valid for the "
@@ -445,41 +509,46 @@ def run_gpu(args, w):
                                  "S_at_last_sync": float(tt["S"][-1]) if len(tt["S"]) else None,
                                  "wire_bytes_per_node": stt.wire_bytes_per_node,
                                  "wire_bytes_total": stt.wire_bytes_total}
-        full_pn, full_tot = abi.adpsgd_wire_bytes(n, P, w.K, False)
+        full_pn, full_tot = abi.adpsgd_wire_bytes(n, P_total, w.K, False)
         comparison["fullsgd"] = {"p": 1, "rounds": w.K, "wire_bytes_per_node": full_pn, "wire_bytes_total": full_tot}
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu:
-        r, dt, sample = oracle_sample(w)
-        cpu = {"value": r, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": sample}
+        cpu = cpu_baseline(w)
     ctx.close()
+    k1_traffic, k1_traffic_how = recorded_traffic("local_step_kernel", w.name, k1_bytes)
+    k2_traffic, k2_traffic_how = recorded_traffic("average_kernel", w.name, k2_bytes)
+    ks_traffic, ks_traffic_how = recorded_traffic("sync_step_kernel", w.name, k1_bytes)
 
     if rank == 0:
+        parallelism = "one GPU" if world == 1 else (
+            f"columns split over {world} ranks (rank 0 holds {P} of {P_total}); 16 bytes exchanged per sync")
         line = {
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
-            "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
+            "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True, "scaling": "strong",
             "vs_baseline": None, "dtype": "f32", "data": "synthetic",
-            "config": {"workload": w.name, "n": n, "P": P, "K": w.K, "schedule": f"ADPSGD p_init={w.p_init} K_s={w.K_s}",
+            "config": {"workload": w.name, "n": n, "P": P_total, "K": w.K,
+                       "schedule": f"ADPSGD p_init={w.p_init} K_s={w.K_s}",
                        "rounds_per_step": rounds[-1] if rounds else None,
-                       "l2": "inputs larger than L2 (x, v = %.0f MB)" % (8 * n * P / 1e6),
-                       "parallelism": f"independent problem per rank x{world}"},
+                       "l2": "inputs larger than L2 (x, v = %.0f MB per rank)" % (8 * n * P / 1e6),
+                       "parallelism": parallelism},
             "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
                     "last_step": e2e_phases},
             "gpu_launches": launches,
             "roofline": {"kernel": "local_step_kernel", "bound": "hbm", "achieved": k1_gbs, "peak": peak,
                          "peak_kind": peak_kind, "unit": "GB/s", "frac": k1_gbs / peak,
                          "bytes_per_launch": k1_bytes, "ms_per_launch": k1_ms,
-                         "traffic": recorded_traffic("local_step_kernel", w.name)},
+                         "traffic": k1_traffic, "traffic_source": k1_traffic_how},
             "avg_variance": {"kernel": "average_kernel", "bound": "hbm", "achieved": k2_gbs,
                              "peak": peak, "unit": "GB/s", "frac": k2_gbs / peak, "bytes_per_launch": k2_bytes,
                              "ms_per_launch": k2_ms, "launches": kt2["average_launches"],
                              "timed": "alone, each launch right after a local step",
-                             "traffic": recorded_traffic("average_kernel", w.name)},
+                             "traffic": k2_traffic, "traffic_source": k2_traffic_how},
             "sync_step": None if ks_ms is None else {
                 "kernel": "sync_step_kernel", "bound": "hbm", "achieved": ks_gbs, "peak": peak, "unit": "GB/s",
                 "frac": ks_gbs / peak, "bytes_per_launch": k1_bytes, "ms_per_launch": ks_ms,
                 "launches": kt["sync_step_launches"], "average_launches_in_run": kt["average_launches"],
-                "traffic": recorded_traffic("sync_step_kernel", w.name),
+                "traffic": ks_traffic, "traffic_source": ks_traffic_how,
                 "note": "the local step of each sync iteration fused with its averaging (x not written "
                         "and read back in between); 16 n P + 8 P bytes, the local step's"},
             "local_step_rp_per_s": n * P / (k1_ms / 1000.0),
@@ -650,7 +719,7 @@ def main():
     ap.add_argument("--steps", type=int, default=5)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=["gb300", "reference"], default="gb300")
-    ap.add_argument("--workload", default="resnet18-n8")
+    ap.add_argument("--workload", default=DEFAULT_WORKLOAD)
     ap.add_argument("--iters", type=int, default=None,
                     help="override the workload's iteration count (profiling captures only)")
     ap.add_argument("--no-e2e", action="store_true")

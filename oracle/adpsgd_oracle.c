@@ -277,6 +277,8 @@ void orc_to_bf16_array(const float* in, uint16_t* out, int64_t m)
 /* stream with tag 1, rounded to bf16.                                       */
 void orc_noise_bf16(uint64_t seed, int32_t n, int64_t P, uint16_t* out)
 {
+    /* rows are independent: one host thread per row (OpenMP) */
+    #pragma omp parallel for schedule(static)
     for (int32_t i = 0; i < n; ++i)
         for (int64_t j = 0; j < P; ++j) {
             float z[4];
