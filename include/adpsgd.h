@@ -45,7 +45,8 @@ typedef enum {
     ADPSGD_E_CUDA = -3,    /* a CUDA runtime call failed (see adpsgd_last_error) */
     ADPSGD_E_TIMEOUT = -4, /* a bounded host wait ran out; the work may still be in flight */
     ADPSGD_E_NOMEM = -5,   /* the context's own scratch could not be allocated */
-    ADPSGD_E_STATE = -6    /* call not valid in the current state (e.g. no noise tensor) */
+    ADPSGD_E_STATE = -6,   /* call not valid in the current state (e.g. no noise tensor) */
+    ADPSGD_E_PEER = -7     /* the shard exchange (adpsgd_shard.gather) reported a failure */
 } adpsgd_status;
 
 /* Opaque context: borrowed pointers to x, v, h, c (and the noise tensor),
@@ -250,6 +251,52 @@ int adpsgd_state_init(const adpsgd_schedule* sched, adpsgd_state* state);
  * E_CUDA.  After an error the state is not resumable (restore a checkpoint). */
 int adpsgd_run(adpsgd_ctx* ctx, const adpsgd_schedule* sched, adpsgd_state* state, int64_t k_end,
                adpsgd_trace* trace, adpsgd_stats* stats);
+
+/* Column sharding: one problem split by columns over g processes (one per GPU).
+ *
+ * The local step is elementwise and the averaging reduces over replicas column by column, so a
+ * problem can be cut into contiguous column ranges: shard r holds x and v as [n, P_r] (its
+ * columns of every replica), its slice of h and c, and of the bf16 noise tensor.  Each shard runs
+ * the same schedule.  At every sync the only exchange is the shard's two fp64 partial sums
+ * (D and the loss; Algorithm 2's S_k line needs their totals): `gather` collects them from every
+ * shard, and every shard adds them in shard order starting from 0, so all shards see the same S
+ * and take the same decisions (16 bytes per shard per sync; no parameter traffic).
+ *
+ * gather(local, count, gathered, user) must place every shard's `count` doubles in shard order,
+ * gathered[r * count + t] = local of shard r, and return 0 (nonzero: ADPSGD_E_PEER).  It is
+ * called from the thread that called the library, on every shard at the same syncs.  With
+ * shards == 1 it may be NULL.
+ *
+ * The noise of global column col0 + j is drawn with Philox block (col0 + j) div 4, so a sharded
+ * run gives every column the same x and v as the unsharded run, bit for bit; D and the loss
+ * differ from the unsharded run's only in the order of their fp64 additions. */
+typedef int (*adpsgd_gather_fn)(const double* local, int64_t count, double* gathered, void* user);
+
+typedef struct {
+    int32_t shards;          /* g >= 1 */
+    int32_t index;           /* this shard, 0 <= index < shards */
+    int64_t col0;            /* global column of this shard's first column; a multiple of 4 */
+    int64_t P_total;         /* columns of the whole problem (wire accounting); >= col0 + P */
+    adpsgd_gather_fn gather; /* the exchange (see above) */
+    void* user;              /* passed to gather */
+} adpsgd_shard;
+
+/* Make ctx one shard of a column-split problem (before its first step).  From then on the sums
+ * that adpsgd_run, adpsgd_average_and_variance and adpsgd_variance report (and the per-iteration
+ * variance record) are the totals over all shards, and the wire accounting uses P_total.
+ * Errors: E_INVAL (shards < 1, index out of range, col0 not a multiple of 4 or negative,
+ * P_total < col0 + P, (col0 + P) / 4 >= 2^32, gather NULL with shards > 1). */
+int adpsgd_set_shard(adpsgd_ctx* ctx, const adpsgd_shard* shard);
+
+/* The exchange alone, for tests and for callers that run their own averaging (pure host code):
+ * gathers `count` doubles from every shard through shard->gather and writes their sums in shard
+ * order, out[t] = ((0 + local_0[t]) + local_1[t]) + ...  Errors: E_INVAL, E_PEER. */
+int adpsgd_shard_combine(const adpsgd_shard* shard, const double* local, int64_t count, double* out);
+
+/* The bf16 noise tensor of one shard: columns [col0, col0 + P) of the [n, P_total] tensor that
+ * adpsgd_noise_fill_bf16 fills, as an [n, P] array.  col0 a multiple of 4.  Enqueued only.
+ * Errors: as adpsgd_noise_fill_bf16, and E_INVAL for col0. */
+int adpsgd_noise_fill_bf16_shard(uint64_t seed, int32_t n, int64_t P, int64_t col0, uint16_t* out, void* stream);
 
 /* The period rule alone (Algorithm 2, after the sync at iteration k; pure host code):
  * warm-up (k < K_w) and kind 0 leave the state unchanged; k < K_s: m += 1,

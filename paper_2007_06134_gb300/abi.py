@@ -17,7 +17,7 @@ from . import build as _build
 _lock = threading.Lock()
 _lib = None
 
-OK, E_INVAL, E_ALIGN, E_CUDA, E_TIMEOUT, E_NOMEM, E_STATE = 0, -1, -2, -3, -4, -5, -6
+OK, E_INVAL, E_ALIGN, E_CUDA, E_TIMEOUT, E_NOMEM, E_STATE, E_PEER = 0, -1, -2, -3, -4, -5, -6, -7
 NOISE_PHILOX, NOISE_BF16 = 0, 1
 CPSGD, ADPSGD, PIECEWISE = 0, 1, 2
 PHASE_CONSTANT, PHASE_WARMUP, PHASE_SAMPLING, PHASE_ADAPTING = 0, 1, 2, 3
@@ -26,7 +26,7 @@ PHASE_CONSTANT, PHASE_WARMUP, PHASE_SAMPLING, PHASE_ADAPTING = 0, 1, 2, 3
 class AdpsgdError(RuntimeError):
     def __init__(self, status: int, where: str):
         self.status = status
-        detail = last_error() if status == E_CUDA or status == E_TIMEOUT else ""
+        detail = last_error() if status in (E_CUDA, E_TIMEOUT, E_PEER) else ""
         super().__init__(f"{where}: {strerror(status)} ({status}){': ' + detail if detail else ''}")
 
 
@@ -72,6 +72,15 @@ class KernelTiming(C.Structure):
                 ("sync_step_ms", C.c_double), ("sync_step_launches", C.c_int64)]
 
 
+# int gather(const double* local, int64_t count, double* gathered, void* user)
+GATHER_FN = C.CFUNCTYPE(C.c_int, C.POINTER(C.c_double), C.c_int64, C.POINTER(C.c_double), C.c_void_p)
+
+
+class Shard(C.Structure):
+    _fields_ = [("shards", C.c_int32), ("index", C.c_int32), ("col0", C.c_int64), ("P_total", C.c_int64),
+                ("gather", GATHER_FN), ("user", C.c_void_p)]
+
+
 _P = C.c_void_p
 _SIGS = {
     "adpsgd_init": (C.c_int, [C.POINTER(Config), _P, _P, _P, _P, _P, _P, C.POINTER(_P)]),
@@ -91,6 +100,9 @@ _SIGS = {
     "adpsgd_philox_fill": (C.c_int, [C.c_uint64, C.c_uint32, C.c_int32, C.c_int64, C.c_int64, _P, _P]),
     "adpsgd_noise_fill_f32": (C.c_int, [C.c_uint64, C.c_uint32, C.c_int32, C.c_int64, C.c_int64, _P, _P]),
     "adpsgd_noise_fill_bf16": (C.c_int, [C.c_uint64, C.c_int32, C.c_int64, _P, _P]),
+    "adpsgd_set_shard": (C.c_int, [_P, C.POINTER(Shard)]),
+    "adpsgd_shard_combine": (C.c_int, [C.POINTER(Shard), C.POINTER(C.c_double), C.c_int64, C.POINTER(C.c_double)]),
+    "adpsgd_noise_fill_bf16_shard": (C.c_int, [C.c_uint64, C.c_int32, C.c_int64, C.c_int64, _P, _P]),
     "adpsgd_copy_h2d": (C.c_int, [_P, _P, C.c_int64, _P]),
     "adpsgd_copy_d2h": (C.c_int, [_P, _P, C.c_int64, _P]),
     "adpsgd_kernel_times": (C.c_int, [_P, C.POINTER(KernelTiming)]),
@@ -217,6 +229,28 @@ def adpsgd_init(cfg: Config, x, v, h, c, noise_bf16=None, stream=None) -> Contex
     return Context(out.value, (x, v, h, c, noise_bf16))
 
 
+def make_shard(shards: int, index: int, col0: int, P_total: int, gather=None) -> Shard:
+    """gather: a GATHER_FN (or None with one shard); the struct keeps a reference to it."""
+    sh = Shard(shards, index, col0, P_total, gather if gather is not None else GATHER_FN(), None)
+    sh._keep = gather
+    return sh
+
+
+def adpsgd_set_shard(ctx: Context, shard: Shard) -> None:
+    _check(load().adpsgd_set_shard(ctx.handle, C.byref(shard)), "adpsgd_set_shard")
+    ctx._shard = shard  # the context calls shard.gather until it is destroyed
+
+
+def adpsgd_shard_combine(shard: Shard, local):
+    """Every shard's values through shard.gather, summed in shard order (pure host code)."""
+    import numpy as np
+    loc = np.ascontiguousarray(local, dtype=np.float64)
+    out = np.zeros_like(loc)
+    _check(load().adpsgd_shard_combine(C.byref(shard), loc.ctypes.data_as(C.POINTER(C.c_double)), loc.size,
+                                       out.ctypes.data_as(C.POINTER(C.c_double))), "adpsgd_shard_combine")
+    return out
+
+
 def adpsgd_local_steps(ctx: Context, k0: int, lr) -> None:
     lr = list(lr)
     arr = (C.c_float * max(1, len(lr)))(*lr)
@@ -328,6 +362,11 @@ def adpsgd_noise_fill_f32(seed: int, tag: int, n: int, P: int, k: int, out, stre
 def adpsgd_noise_fill_bf16(seed: int, n: int, P: int, out, stream=None) -> None:
     _check(load().adpsgd_noise_fill_bf16(seed & 0xFFFFFFFFFFFFFFFF, n, P, _ptr(out), _stream(stream)),
            "adpsgd_noise_fill_bf16")
+
+
+def adpsgd_noise_fill_bf16_shard(seed: int, n: int, P: int, col0: int, out, stream=None) -> None:
+    _check(load().adpsgd_noise_fill_bf16_shard(seed & 0xFFFFFFFFFFFFFFFF, n, P, col0, _ptr(out), _stream(stream)),
+           "adpsgd_noise_fill_bf16_shard")
 
 
 def _nbytes(t, nbytes):

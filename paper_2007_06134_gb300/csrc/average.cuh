@@ -173,16 +173,17 @@ __device__ void redo_group(const AvgParams& p, int64_t q, float nf, double& accD
             for (int i = 0; i < p.n; ++i) p.x[(int64_t)i * p.P + W * q + r] = xbar[r];
 }
 
-// The end of a persistent averaging kernel: each block leaves its fp64 partials of D and the loss;
-// the last block to finish (an atomic ticket, no inter-block wait) adds them in block order into
-// out[0] = D and out[1] = loss / 2, and resets the ticket.  Deterministic for a given grid.
-template <bool LOSS>
-__device__ __forceinline__ void finish_sums(const AvgParams& p, double accD, double accL)
+// The end of a persistent averaging kernel of THREADS-thread blocks: each block leaves its fp64
+// partials of D and the loss; the last block to finish (an atomic ticket, no inter-block wait)
+// adds them in block order into out[0] = D and out[1] = loss / 2, and resets the ticket.
+// Deterministic for a given grid.
+template <bool LOSS, int THREADS>
+__device__ __forceinline__ void finish_sums_n(const AvgParams& p, double accD, double accL)
 {
-    __shared__ double shared[kThreads / 32];
+    __shared__ double shared[THREADS / 32];
     __shared__ unsigned int ticket;
-    const double bD = block_sum(accD, shared);
-    const double bL = LOSS ? block_sum(accL, shared) : 0.0;
+    const double bD = block_sum<THREADS>(accD, shared);
+    const double bL = LOSS ? block_sum<THREADS>(accL, shared) : 0.0;
     if (threadIdx.x == 0) {
         p.partials[blockIdx.x] = bD;
         p.partials[gridDim.x + blockIdx.x] = bL;
@@ -194,17 +195,23 @@ __device__ __forceinline__ void finish_sums(const AvgParams& p, double accD, dou
     // The last block: every other block's partials are visible (fence before each increment).
     __threadfence();
     double d = 0.0, l = 0.0;
-    for (int b = threadIdx.x; b < (int)gridDim.x; b += kThreads) {
+    for (int b = threadIdx.x; b < (int)gridDim.x; b += THREADS) {
         d += __ldcg(p.partials + b);
         if (LOSS) l += __ldcg(p.partials + gridDim.x + b);
     }
-    d = block_sum(d, shared);
-    if (LOSS) l = block_sum(l, shared);
+    d = block_sum<THREADS>(d, shared);
+    if (LOSS) l = block_sum<THREADS>(l, shared);
     if (threadIdx.x == 0) {
         p.out[0] = d;
         p.out[1] = 0.5 * l;
         *p.counter = 0u;
     }
+}
+
+template <bool LOSS>
+__device__ __forceinline__ void finish_sums(const AvgParams& p, double accD, double accL)
+{
+    finish_sums_n<LOSS, kThreads>(p, accD, accL);
 }
 
 }  // namespace

@@ -31,7 +31,9 @@ __device__ __forceinline__ void sgd_update(float& x, float& v, float h, float c,
 
 __device__ __forceinline__ float bf16_bits_to_float(uint32_t bits16) { return __uint_as_float(bits16 << 16); }
 
-// Fixed-order block sum over a block of kThreads threads; the result is valid in thread 0.
+// Fixed-order block sum over a block of THREADS threads (shared: THREADS / 32 doubles); the
+// result is valid in thread 0.
+template <int THREADS = kThreads>
 __device__ __forceinline__ double block_sum(double v, double* shared)
 {
 #pragma unroll
@@ -41,7 +43,7 @@ __device__ __forceinline__ double block_sum(double v, double* shared)
     __syncthreads();
     double total = 0.0;
     if (threadIdx.x == 0)
-        for (int w = 0; w < kThreads / 32; ++w) total += shared[w];
+        for (int w = 0; w < THREADS / 32; ++w) total += shared[w];
     __syncthreads();
     return total;
 }

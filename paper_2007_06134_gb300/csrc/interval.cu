@@ -33,6 +33,7 @@ struct IntervalParams {
     int64_t Q;  // ceil(P / 4)
     int32_t n;
     uint32_t k0;
+    uint32_t q0;  // Philox block of column 0
     int32_t m;
     float mu, wd, sigma;
     double* partials;
@@ -134,7 +135,7 @@ __global__ void __launch_bounds__(kTileGroups * kMaxReplicas) interval_kernel(co
                 if (BF16) {
                     z[0] = zb[0]; z[1] = zb[1]; z[2] = zb[2]; z[3] = zb[3];
                 } else {
-                    const float4 z4 = normals4(p.keys, (uint32_t)q, (uint32_t)i, p.k0 + (uint32_t)s, 0u);
+                    const float4 z4 = normals4(p.keys, (uint32_t)q + p.q0, (uint32_t)i, p.k0 + (uint32_t)s, 0u);
                     z[0] = z4.x; z[1] = z4.y; z[2] = z4.z; z[3] = z4.w;
                 }
                 const float gamma = p.gamma[s];
@@ -270,6 +271,7 @@ cudaError_t launch_interval(const IntervalArgs& a, cudaStream_t stream)
     p.Q = (a.P + 3) / 4;
     p.n = a.n;
     p.k0 = a.k0;
+    p.q0 = a.q0;
     p.m = a.m;
     p.mu = a.mu;
     p.wd = a.wd;

@@ -28,6 +28,7 @@ struct LocalStepArgs {
     int32_t n;
     int64_t P;
     uint32_t k;
+    uint32_t q0;  // Philox block of column 0 (a shard's column offset / 4; 0 unsharded)
     float gamma, mu, wd, sigma;
 };
 cudaError_t launch_local_step(const LocalStepArgs& a, cudaStream_t stream);
@@ -66,6 +67,7 @@ struct SyncStepArgs {
     int32_t n;
     int64_t P;
     uint32_t k;
+    uint32_t q0;       // Philox block of column 0
     float gamma, mu, wd, sigma;
     bool loss;
     double* partials;  // 2 * grid doubles
@@ -100,6 +102,7 @@ struct IntervalArgs {
     int32_t n;
     int64_t P;
     uint32_t k0;
+    uint32_t q0;         // Philox block of column 0
     int32_t m;
     const float* gamma;  // host array of m step sizes
     float mu, wd, sigma;
@@ -119,7 +122,8 @@ cudaError_t launch_philox_fill(uint64_t seed, uint32_t tag, int32_t n, int64_t n
                                uint32_t* out, cudaStream_t stream);
 cudaError_t launch_noise_f32(uint64_t seed, uint32_t tag, int32_t n, int64_t P, uint32_t k,
                              float* out, cudaStream_t stream);
-cudaError_t launch_noise_bf16(uint64_t seed, int32_t n, int64_t P, uint16_t* out,
+// The bf16 noise tensor of columns [4 q0, 4 q0 + P) of the whole problem.
+cudaError_t launch_noise_bf16(uint64_t seed, int32_t n, int64_t P, uint32_t q0, uint16_t* out,
                               cudaStream_t stream);
 
 }  // namespace adpsgd

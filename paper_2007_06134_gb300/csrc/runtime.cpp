@@ -39,6 +39,35 @@ bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) ==
 
 constexpr int64_t kMaxK = int64_t(1) << 32;  // the step index is one 32-bit Philox counter word
 
+int check_shard(const adpsgd_shard* sh)
+{
+    if (sh == nullptr || sh->shards < 1 || sh->index < 0 || sh->index >= sh->shards) return ADPSGD_E_INVAL;
+    if (sh->col0 < 0 || sh->col0 % 4 != 0 || sh->P_total < sh->col0) return ADPSGD_E_INVAL;
+    if (sh->shards > 1 && sh->gather == nullptr) return ADPSGD_E_INVAL;
+    return ADPSGD_OK;
+}
+
+// Every shard's `count` doubles through shard->gather, added in shard order from 0.
+int shard_combine(const adpsgd_shard* sh, const double* local, int64_t count, double* out)
+{
+    if (sh->gather == nullptr) {  // a single shard
+        for (int64_t t = 0; t < count; ++t) out[t] = 0.0 + local[t];
+        return ADPSGD_OK;
+    }
+    std::vector<double> all((size_t)count * (size_t)sh->shards, 0.0);
+    const int rc = sh->gather(local, count, all.data(), sh->user);
+    if (rc != 0) {
+        g_last_error = "shard exchange failed with code " + std::to_string(rc);
+        return ADPSGD_E_PEER;
+    }
+    for (int64_t t = 0; t < count; ++t) {
+        double total = 0.0;
+        for (int32_t r = 0; r < sh->shards; ++r) total += all[(size_t)r * (size_t)count + (size_t)t];
+        out[t] = total;
+    }
+    return ADPSGD_OK;
+}
+
 }  // namespace
 
 struct TimedLaunch {
@@ -73,6 +102,10 @@ struct adpsgd_ctx {
     int64_t launches[4] = {0, 0, 0, 0};
     int64_t timed_launches[4] = {0, 0, 0, 0};
     bool force_incomplete = false;
+    // column sharding (adpsgd_set_shard): the Philox block of column 0 and the exchange
+    uint32_t q0 = 0;
+    bool sharded = false;
+    adpsgd_shard shard{};
 };
 
 namespace {
@@ -188,6 +221,7 @@ int local_step(adpsgd_ctx* ctx, int64_t k, float gamma)
     a.n = ctx->cfg.n;
     a.P = ctx->cfg.P;
     a.k = (uint32_t)k;
+    a.q0 = ctx->q0;
     a.gamma = gamma;
     a.mu = ctx->cfg.momentum;
     a.wd = ctx->cfg.weight_decay;
@@ -245,6 +279,23 @@ int average(adpsgd_ctx* ctx, bool write_back, bool loss)
     return wait_event(ctx, ctx->done);
 }
 
+// D and the loss of the last averaging (ctx->h_out): this context's own sums, or for a shard of a
+// column-split problem the totals over all shards in shard order.
+int sync_sums(adpsgd_ctx* ctx, double* D, double* loss)
+{
+    if (!ctx->sharded) {
+        *D = ctx->h_out[0];
+        *loss = ctx->h_out[1];
+        return ADPSGD_OK;
+    }
+    double total[2];
+    const int st = shard_combine(&ctx->shard, ctx->h_out, 2, total);
+    if (st != ADPSGD_OK) return st;
+    *D = total[0];
+    *loss = total[1];
+    return ADPSGD_OK;
+}
+
 // Enqueue one fused interval: m local steps from step k0 (step sizes gamma[0..m)) and, if
 // `average`, the averaging with the copy of its sums and ctx->done.
 int interval(adpsgd_ctx* ctx, int64_t k0, int32_t m, const float* gamma, bool average, bool loss)
@@ -259,6 +310,7 @@ int interval(adpsgd_ctx* ctx, int64_t k0, int32_t m, const float* gamma, bool av
     a.n = ctx->cfg.n;
     a.P = ctx->cfg.P;
     a.k0 = (uint32_t)k0;
+    a.q0 = ctx->q0;
     a.m = m;
     a.gamma = gamma;
     a.mu = ctx->cfg.momentum;
@@ -294,6 +346,7 @@ int sync_step_enqueue(adpsgd_ctx* ctx, int64_t k, float gamma, bool loss)
     a.n = ctx->cfg.n;
     a.P = ctx->cfg.P;
     a.k = (uint32_t)k;
+    a.q0 = ctx->q0;
     a.gamma = gamma;
     a.mu = ctx->cfg.momentum;
     a.wd = ctx->cfg.weight_decay;
@@ -418,6 +471,7 @@ const char* adpsgd_strerror(int status)
     case ADPSGD_E_TIMEOUT: return "bounded wait timed out";
     case ADPSGD_E_NOMEM: return "out of memory";
     case ADPSGD_E_STATE: return "invalid state for this call";
+    case ADPSGD_E_PEER: return "the shard exchange failed";
     default: return "unknown status";
     }
 }
@@ -526,8 +580,11 @@ int adpsgd_average_and_variance(adpsgd_ctx* ctx, double* D_out, double* loss_out
     if (loss_out != nullptr && !ctx->cfg.want_loss) return ADPSGD_E_STATE;
     int st = average(ctx, true, loss_out != nullptr);
     if (st != ADPSGD_OK) return st;
-    *D_out = ctx->h_out[0];
-    if (loss_out != nullptr) *loss_out = ctx->h_out[1];
+    double D = 0.0, loss = 0.0;
+    st = sync_sums(ctx, &D, &loss);
+    if (st != ADPSGD_OK) return st;
+    *D_out = D;
+    if (loss_out != nullptr) *loss_out = loss;
     return ADPSGD_OK;
 }
 
@@ -536,7 +593,10 @@ int adpsgd_variance(adpsgd_ctx* ctx, double* D_out)
     if (ctx == nullptr || D_out == nullptr) return ADPSGD_E_INVAL;
     int st = average(ctx, false, false);
     if (st != ADPSGD_OK) return st;
-    *D_out = ctx->h_out[0];
+    double D = 0.0, loss = 0.0;
+    st = sync_sums(ctx, &D, &loss);
+    if (st != ADPSGD_OK) return st;
+    *D_out = D;
     return ADPSGD_OK;
 }
 
@@ -643,8 +703,11 @@ int adpsgd_run(adpsgd_ctx* ctx, const adpsgd_schedule* sched, adpsgd_state* stat
                     st = wait_event(ctx, ctx->done);
                 }
                 if (st != ADPSGD_OK) return st;
+                double D = 0.0, L = 0.0;
+                st = sync_sums(ctx, &D, &L);
+                if (st != ADPSGD_OK) return st;
                 const int64_t ks = k + m - 1;
-                const double S = ctx->h_out[0] / (double)ctx->cfg.n;
+                const double S = D / (double)ctx->cfg.n;
                 const int32_t phase = rule(sched, state, ks, S, (double)gam[m - 1]);
                 if (trace != nullptr && trace->len < trace->cap) {
                     const int64_t t = trace->len;
@@ -652,7 +715,7 @@ int adpsgd_run(adpsgd_ctx* ctx, const adpsgd_schedule* sched, adpsgd_state* stat
                     trace->p[t] = state->p;
                     trace->S[t] = S;
                     trace->C2[t] = state->C2;
-                    trace->loss[t] = loss ? ctx->h_out[1] : 0.0;
+                    trace->loss[t] = loss ? L : 0.0;
                     trace->phase[t] = phase;
                     trace->len = t + 1;
                 }
@@ -695,7 +758,10 @@ int adpsgd_run(adpsgd_ctx* ctx, const adpsgd_schedule* sched, adpsgd_state* stat
             st = wait_event(ctx, ctx->done);
         }
         if (st != ADPSGD_OK) return st;
-        const double S = ctx->h_out[0] / (double)ctx->cfg.n;
+        double D = 0.0, L = 0.0;
+        st = sync_sums(ctx, &D, &L);
+        if (st != ADPSGD_OK) return st;
+        const double S = D / (double)ctx->cfg.n;
         const int32_t phase = rule(sched, state, k, S, (double)gamma_of(sched, k));
         if (trace != nullptr) {
             if (trace->len < trace->cap) {
@@ -704,7 +770,7 @@ int adpsgd_run(adpsgd_ctx* ctx, const adpsgd_schedule* sched, adpsgd_state* stat
                 trace->p[t] = state->p;
                 trace->S[t] = S;
                 trace->C2[t] = state->C2;
-                trace->loss[t] = loss ? ctx->h_out[1] : 0.0;
+                trace->loss[t] = loss ? L : 0.0;
                 trace->phase[t] = phase;
                 trace->len = t + 1;
             }
@@ -721,15 +787,23 @@ int adpsgd_run(adpsgd_ctx* ctx, const adpsgd_schedule* sched, adpsgd_state* stat
             if (e != cudaSuccess) return cuda_fail(e, "variance copy");
             st = wait_event(ctx, ctx->done);
             if (st != ADPSGD_OK) return st;
-            for (int64_t k = k_first; k < last; ++k) trace->var[k] = slots[2 * (size_t)(k - k_first)] / (double)ctx->cfg.n;
+            std::vector<double> D((size_t)(last - k_first));
+            for (int64_t k = k_first; k < last; ++k) D[(size_t)(k - k_first)] = slots[2 * (size_t)(k - k_first)];
+            if (ctx->sharded) {
+                std::vector<double> local = D;
+                st = shard_combine(&ctx->shard, local.data(), (int64_t)local.size(), D.data());
+                if (st != ADPSGD_OK) return st;
+            }
+            for (int64_t k = k_first; k < last; ++k) trace->var[k] = D[(size_t)(k - k_first)] / (double)ctx->cfg.n;
         }
     }
     if (stats != nullptr) {
         stats->rounds = state->rounds;
         stats->equiv_period = state->rounds > 0 ? (double)state->k_next / (double)state->rounds : 0.0;
         double total = 0.0;
-        wire(ctx->cfg.n, ctx->cfg.P, state->rounds, true, &stats->wire_bytes_per_node, &stats->wire_bytes_total);
-        wire(ctx->cfg.n, ctx->cfg.P, state->k_next, false, &stats->fullsgd_wire_bytes_per_node, &total);
+        const int64_t P_all = ctx->sharded ? ctx->shard.P_total : ctx->cfg.P;
+        wire(ctx->cfg.n, P_all, state->rounds, true, &stats->wire_bytes_per_node, &stats->wire_bytes_total);
+        wire(ctx->cfg.n, P_all, state->k_next, false, &stats->fullsgd_wire_bytes_per_node, &total);
         stats->local_step_launches = ctx->launches[0] - launches0[0];
         stats->average_launches = ctx->launches[1] - launches0[1];
         stats->interval_launches = ctx->launches[2] - launches0[2];
@@ -818,8 +892,36 @@ int adpsgd_noise_fill_bf16(uint64_t seed, int32_t n, int64_t P, uint16_t* out, v
     if (out == nullptr || n < 0 || P < 0 || P > (int64_t(1) << 34)) return ADPSGD_E_INVAL;
     if ((int64_t)n * P > (int64_t(1) << 40)) return ADPSGD_E_INVAL;
     if (!aligned16(out)) return ADPSGD_E_ALIGN;
-    cudaError_t e = adpsgd::launch_noise_bf16(seed, n, P, out, static_cast<cudaStream_t>(stream));
+    cudaError_t e = adpsgd::launch_noise_bf16(seed, n, P, 0u, out, static_cast<cudaStream_t>(stream));
     return e == cudaSuccess ? ADPSGD_OK : cuda_fail(e, "bf16 noise fill");
+}
+
+int adpsgd_noise_fill_bf16_shard(uint64_t seed, int32_t n, int64_t P, int64_t col0, uint16_t* out, void* stream)
+{
+    if (out == nullptr || n < 0 || P < 0 || P > (int64_t(1) << 34)) return ADPSGD_E_INVAL;
+    if (col0 < 0 || col0 % 4 != 0 || (col0 + P + 3) / 4 > kMaxK) return ADPSGD_E_INVAL;
+    if ((int64_t)n * P > (int64_t(1) << 40)) return ADPSGD_E_INVAL;
+    if (!aligned16(out)) return ADPSGD_E_ALIGN;
+    cudaError_t e = adpsgd::launch_noise_bf16(seed, n, P, (uint32_t)(col0 / 4), out, static_cast<cudaStream_t>(stream));
+    return e == cudaSuccess ? ADPSGD_OK : cuda_fail(e, "bf16 noise fill");
+}
+
+int adpsgd_set_shard(adpsgd_ctx* ctx, const adpsgd_shard* shard)
+{
+    if (ctx == nullptr || check_shard(shard) != ADPSGD_OK) return ADPSGD_E_INVAL;
+    if (shard->P_total < shard->col0 + ctx->cfg.P) return ADPSGD_E_INVAL;
+    if ((shard->col0 + ctx->cfg.P + 3) / 4 > kMaxK) return ADPSGD_E_INVAL;  // Philox blocks are 32-bit words
+    ctx->shard = *shard;
+    ctx->sharded = true;
+    ctx->q0 = (uint32_t)(shard->col0 / 4);
+    return ADPSGD_OK;
+}
+
+int adpsgd_shard_combine(const adpsgd_shard* shard, const double* local, int64_t count, double* out)
+{
+    if (check_shard(shard) != ADPSGD_OK || count < 0 || (count > 0 && (local == nullptr || out == nullptr)))
+        return ADPSGD_E_INVAL;
+    return shard_combine(shard, local, count, out);
 }
 
 namespace {

@@ -21,7 +21,7 @@ def test_library_exports_every_header_entry_point():
 
 
 def test_strerror_covers_every_status():
-    for st in (abi.OK, abi.E_INVAL, abi.E_ALIGN, abi.E_CUDA, abi.E_TIMEOUT, abi.E_NOMEM, abi.E_STATE):
+    for st in (abi.OK, abi.E_INVAL, abi.E_ALIGN, abi.E_CUDA, abi.E_TIMEOUT, abi.E_NOMEM, abi.E_STATE, abi.E_PEER):
         assert abi.strerror(st) and abi.strerror(st) != "unknown status"
     assert abi.strerror(12345) == "unknown status"
 

@@ -25,6 +25,7 @@ STRUCTS = {
     "adpsgd_trace": abi.Trace,
     "adpsgd_stats": abi.Stats,
     "adpsgd_kernel_timing": abi.KernelTiming,
+    "adpsgd_shard": abi.Shard,
 }
 
 

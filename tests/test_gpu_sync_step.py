@@ -81,6 +81,35 @@ def test_noise_modes_weight_decay_and_no_loss(bf16, wd, loss):
     _against_oracle(r, loss=loss)
 
 
+@pytest.mark.parametrize("n", [3, 4, 6, 8])
+def test_pipelined_form_with_several_groups_per_thread(n):
+    # With Philox noise and 3..8 replicas the fused step runs the pipelined form (asynchronous
+    # copies into shared memory, refilled for the next group while a group is stepped and
+    # averaged).  At 2^20 + 148 columns every thread of its persistent grid takes two or three
+    # groups, so the refills are consumed: whole runs bit-exact against the oracle.
+    P, K = (1 << 20) + 4 * 37, 12
+    w = inputs.WORKLOADS["resnet18-n8"]
+    h, c = inputs.draw_h(P, w.h_dist, 8), inputs.draw_c(P, 1.0, 8)
+    x, v = inputs.random_state(n, P, 8)
+    xd, vd = dev(x), dev(v)
+    cfg = abi.make_config(n, P, momentum=0.9, weight_decay=5e-4, noise_sigma=0.8, seed=w.seed, fuse_sync_step=True)
+    sched = abi.make_schedule(abi.ADPSGD, K, 2, K_s=4, lr0=0.1)
+    tr = abi.TraceBuffers(K + 1)
+    with abi.adpsgd_init(cfg, xd, vd, dev(h), dev(c)) as ctx:
+        st = abi.adpsgd_run(ctx, sched, abi.adpsgd_state_init(sched), trace=tr)
+    assert st.sync_step_launches > 0
+    spec = O.ScheduleSpec(kind=abi.ADPSGD, K=K, p_init=2, K_s=4, lr0=0.1)
+    otr = O.run(x, v, h, c, spec=spec, seed=w.seed, mu=0.9, wd=5e-4, sigma=0.8, threads=O.host_threads())
+    g = tr.arrays()
+    assert np.array_equal(g["k"], otr.k) and np.array_equal(g["p"], otr.p)
+    for a, b in zip(g["S"], otr.S):
+        assert rel(a, b) < REL
+    for a, b in zip(g["loss"], otr.loss):
+        assert rel(a, b) < REL
+    assert np.array_equal(host(xd).view(np.uint32), x.view(np.uint32))
+    assert np.array_equal(host(vd).view(np.uint32), v.view(np.uint32))
+
+
 def test_fused_equals_unfused_at_a_larger_size():
     args = dict(n=8, P=(1 << 20) + 4 * 11, K=120, kind=abi.ADPSGD, p=4, K_s=30, milestones=(60, 90))
     a = _run(fused=False, **args)
