@@ -61,7 +61,7 @@ typedef struct {
     int32_t noise_mode;      /* ADPSGD_NOISE_PHILOX: z drawn per step from Philox4x32-10;
                                 ADPSGD_NOISE_BF16: z read from a caller tensor [n, P] bf16 */
     int64_t P;               /* parameters per replica, >= 1 */
-    float momentum;          /* mu (Sec. V-A uses 0.9) */
+    float momentum;          /* mu (Sec. IV-A uses 0.9) */
     float weight_decay;      /* wd, added to the gradient as wd * x (0 = off) */
     float noise_sigma;       /* sigma: g = h (x - c) + sigma z */
     int32_t want_loss;       /* nonzero: averaging also returns 1/2 sum_j h_j (xbar_j - c_j)^2 */
@@ -86,7 +86,7 @@ typedef struct {
 } adpsgd_config;
 
 /* Schedules (Algorithm 1: kind 0; Algorithm 2: kind 1; kind 2: a piecewise-constant period,
- * such as the four strategies of Sec. IV-A and the decreasing period of Sec. VI-B). */
+ * such as the four strategies of Sec. III-A and the decreasing period of Sec. V-B). */
 enum { ADPSGD_CPSGD = 0, ADPSGD_ADPSGD = 1, ADPSGD_PIECEWISE = 2 };
 
 typedef struct {
@@ -96,7 +96,7 @@ typedef struct {
     int64_t K_s;             /* Algorithm 2: syncs at iterations k < K_s sample C_2;
                                 must be >= p_init (+ K_w) so that C_2 gets a sample */
     int64_t K_w;             /* warm-up: iterations k < K_w sync every iteration and are
-                                not sampled (Sec. V-B warm-up epoch); 0 = none */
+                                not sampled (Sec. IV-B warm-up epoch); 0 = none */
     double lo, hi;           /* Algorithm 2 thresholds, 0.7 and 1.3 in the paper */
     int32_t p_min, p_max;    /* clamp of p after the rule; p_max = 0: no upper bound */
     double lr0;              /* step size at k = 0 */
@@ -109,7 +109,7 @@ typedef struct {
     int32_t reserved;          /* period_change_k[t] on (increasing k, values >= 1; host arrays) */
     const int64_t* period_change_k;
     const int32_t* period_values;
-    int32_t lr_warmup_steps;   /* step-size warm-up of Sec. V-C (0 = none): on stair
+    int32_t lr_warmup_steps;   /* step-size warm-up of Sec. IV-C (0 = none): on stair
                                   s = min(k div lr_warmup_len, lr_warmup_steps - 1) the step size is
                                   lr0 * (s + 1) before the milestone factors */
     int32_t reserved2;
@@ -138,7 +138,7 @@ typedef struct {
     int32_t* phase;          /* 0 constant, 1 warm-up, 2 sampling, 3 adapting */
     int64_t var_cap;         /* entries of var (0: not recorded) */
     double* var;             /* var[k] = Var[W_k] = D / n at the start of iteration k, k < var_cap
-                                (Sec. III; the series behind V_t of Eq. vt and the weighted variance
+                                (Sec. II-B; the series behind V_t of Eq. vt and the weighted variance
                                 of Eq. metric2).  Costs one variance pass (4 B per replica-param) per
                                 iteration; not available with cfg.fuse_intervals */
 } adpsgd_trace;
@@ -177,14 +177,14 @@ int adpsgd_init(const adpsgd_config* cfg, float* x, float* v, const float* h, co
                 const uint16_t* noise_bf16, void* stream, adpsgd_ctx** out);
 
 /* m local steps of every replica (Algorithm 1 and 2, "updating parameter variables locally";
- * Sec. V-A momentum): for t in [0, m), step k = k0 + t with step size lr[t] (host array):
+ * Sec. IV-A momentum): for t in [0, m), step k = k0 + t with step size lr[t] (host array):
  *   g = h (x - c) + sigma z[i, j, k];  if wd != 0: g += wd x;  v = mu v + g;  x -= lr[t] v
  * each a separately rounded fp32 operation.  z is word (j mod 4) of Philox4x32-10 with counter
  * (j div 4, i, k, 0) and key (seed lo, seed hi), mapped through Box-Muller.  Enqueued only;
  * does not wait.  Errors: E_INVAL (m < 0, k0 < 0, k0 + m > 2^32), E_CUDA. */
 int adpsgd_local_steps(adpsgd_ctx* ctx, int64_t k0, int32_t m, const float* lr);
 
-/* Synchronisation (Algorithm 2 averaging and S_k lines; Sec. III definition of Var[W_k]):
+/* Synchronisation (Algorithm 2 averaging and S_k lines; Sec. II-B definition of Var[W_k]):
  * for every column j, xbar_j = x_0j + (sum_{i>=1} (x_ij - x_0j)) / n in fp32, written back to
  * all n replicas, and *D_out = sum_j sum_i (x_ij - xbar_j)^2 over the pre-average values
  * (n * Var[W]), accumulated in fp64.  If loss_out != NULL (needs cfg.want_loss),
@@ -229,7 +229,7 @@ int adpsgd_average_and_variance_static(float* x, const float* h, const float* c,
                                        double* D_out, double* loss_out, int64_t wait_timeout_ms, void* stream);
 
 /* D = sum_j sum_i (x_ij - xbar_j)^2 without averaging (the per-iteration Var[W_k] of
- * Sec. III and Eq. vt, times n).  Blocks (bounded).  Errors: as above. */
+ * Sec. II-B and Eq. vt, times n).  Blocks (bounded).  Errors: as above. */
 int adpsgd_variance(adpsgd_ctx* ctx, double* D_out);
 
 /* Initial scheduler state of a schedule: k_next 0, cnt 0, p = p_init, C2 0.  Errors: E_INVAL. */
@@ -313,7 +313,7 @@ int adpsgd_gamma(const adpsgd_schedule* sched, int64_t k, float* gamma_out);
 
 /* Bytes a ring allreduce would move per node and in total for `rounds` syncs of P fp32
  * values, 2 (n-1)/n * 4P each (plus 2 (n-1)/n * 4 for the fp32 S_k if with_scalar): the
- * communication Algorithm 2 saves (Sec. V-B).  Errors: E_INVAL. */
+ * communication Algorithm 2 saves (Sec. IV-B).  Errors: E_INVAL. */
 int adpsgd_wire_bytes(int32_t n, int64_t P, int64_t rounds, int32_t with_scalar,
                       double* per_node, double* total);
 

@@ -16,9 +16,9 @@
  *   - The local step of Algorithm 1 (update line) and Algorithm 2 (update line)
  *     on the surrogate objective f(x) = 1/2 sum_j h_j (x_j - c_j)^2, with SGD
  *     momentum and weight decay in the PyTorch 1.0 convention the experiments
- *     used (Sec. V-A: "momentum coefficient 0.9").
+ *     used (Sec. IV-A: "momentum coefficient 0.9").
  *   - Parameter averaging (Algorithm 2, averaging line; Eq. alg1's A_n) and the
- *     inter-replica variance of Sec. III (definition of Var[W_k]) and S_k of
+ *     inter-replica variance of Sec. II-B (definition of Var[W_k]) and S_k of
  *     Algorithm 2, plus the surrogate loss at the average.
  *   - The period rule of Algorithm 2 (cnt, p, C_2; sampling phase k < K_s;
  *     +1 / -1 at 0.7 and 1.3) and Algorithm 1 as the constant-period case.
@@ -38,13 +38,13 @@
  *      fp32 -- equal to (1/n) sum_i x_i in exact arithmetic -- so that the
  *      variance right after averaging is exactly zero (Sec. III-B) and n = 1 is
  *      exactly the identity.
- *   R4 S_k = D / n with D = sum_i ||x_i - xbar||^2 (Sec. III definition of Var).
+ *   R4 S_k = D / n with D = sum_i ||x_i - xbar||^2 (Sec. II-B definition of Var).
  *   R5 RunningAverage = cumulative arithmetic mean of S_k / gamma_k.
  *   R6 p is clamped to [p_min, p_max] (p_max = 0: no upper bound).
  *   R7 the constant-period schedule syncs when cnt reaches p (as Algorithm 2
  *      with adaptation off); Algorithm 1's literal "k mod p == 0" is a flag.
  *   R8 optional warm-up: the first K_w iterations sync every iteration and are
- *      not sampled into C_2 (Sec. V-B).
+ *      not sampled into C_2 (Sec. IV-B).
  */
 #include <math.h>
 #include <stdint.h>
@@ -334,7 +334,7 @@ void orc_local_step(int32_t n, int64_t P, int64_t j0, int64_t j1, float* x, floa
 }
 
 /* ------------------------------------------------------------------------ */
-/* Averaging and variance (Algorithm 2, averaging and S_k lines; Sec. III   */
+/* Averaging and variance (Algorithm 2, averaging and S_k lines; Sec. II-B   */
 /* definition of Var[W_k]) for columns [j0, j1).                             */
 /* xbar_j (fp32, reading R3) is written back to every replica.               */
 /* *D    += sum_j sum_i (x_ij - xbar_j)^2   in fp64 (before the write-back)  */
@@ -387,8 +387,8 @@ double orc_variance(int32_t n, int64_t P, const float* x) { return orc_variance_
 /* ------------------------------------------------------------------------ */
 typedef struct {
     int32_t kind;          /* 0 constant period (Algorithm 1), 1 adaptive (Algorithm 2),
-                              2 piecewise-constant period (the strategies of Sec. IV-A and the
-                              decreasing period of Sec. VI-B) */
+                              2 piecewise-constant period (the strategies of Sec. III-A and the
+                              decreasing period of Sec. V-B) */
     int32_t p_init;        /* constant p, or p_init */
     int64_t K;             /* iterations */
     int64_t K_s;           /* sampling phase: syncs at k < K_s sample C_2 */
@@ -404,7 +404,7 @@ typedef struct {
     int32_t pad;
     const int64_t* period_change_k;
     const int32_t* period_values;
-    int32_t lr_warmup_steps;   /* step-size warm-up (Sec. V-C): gamma = lr0 * (s + 1) on stair s,   */
+    int32_t lr_warmup_steps;   /* step-size warm-up (Sec. IV-C): gamma = lr0 * (s + 1) on stair s,   */
     int32_t pad2;              /* s = min(k div lr_warmup_len, lr_warmup_steps - 1); 0: no warm-up */
     int64_t lr_warmup_len;
 } orc_schedule;
@@ -492,7 +492,7 @@ typedef struct {
     double* loss;    /* surrogate loss at the average */
     int32_t* phase;  /* phase code */
     int64_t cap;     /* capacity of the arrays */
-    double* var;     /* optional: var[k] = Var[W_k] (Sec. III) at the start of iteration k */
+    double* var;     /* optional: var[k] = Var[W_k] (Sec. II-B) at the start of iteration k */
     int64_t var_cap; /* entries of var */
 } orc_trace;
 

@@ -253,7 +253,7 @@ def average_variance(x, h=None, c=None, j0=0, j1=None):
 
 
 def variance(x) -> float:
-    """D = sum_i ||x_i - xbar||^2 without averaging (Sec. III, Var[W_k] times n)."""
+    """D = sum_i ||x_i - xbar||^2 without averaging (Sec. II-B, Var[W_k] times n)."""
     _check_state(x)
     return lib().orc_variance(x.shape[0], x.shape[1], _f32p(x))
 
@@ -276,7 +276,7 @@ class ScheduleSpec:
     milestones: tuple = ()
     literal_phase: int = 0
     period_changes: tuple = ()   # ((k, p), ...) for kind 2
-    lr_warmup_steps: int = 0     # step-size warm-up stairs (Sec. V-C), each lr_warmup_len iterations
+    lr_warmup_steps: int = 0     # step-size warm-up stairs (Sec. IV-C), each lr_warmup_len iterations
     lr_warmup_len: int = 1
     _ms: np.ndarray = field(default=None, repr=False)
     _pk: np.ndarray = field(default=None, repr=False)
@@ -334,7 +334,7 @@ def run(x, v, h, c, *, spec: ScheduleSpec, seed, mu, wd, sigma, noise=None, stat
         k_begin=0, k_end=None, cap=100000, track_variance=False, threads=None,
         chunk=CHUNK_COLUMNS) -> RunTrace:
     """Algorithm 2 (or 1) end to end on the [n, P] arrays, in place; returns the sync trace and,
-    with track_variance, Var[W_k] at the start of every iteration k (Sec. III, Eq. vt).
+    with track_variance, Var[W_k] at the start of every iteration k (Sec. II-B, Eq. vt).
     threads=None runs on one thread in column order; threads=t (e.g. host_threads()) runs the
     chunked all-core form: the same x, v and schedule, D and the loss summed per chunk of `chunk`
     columns in chunk order."""

@@ -185,7 +185,7 @@ def make_schedule(kind, K, p_init, *, K_s=0, K_w=0, lo=0.7, hi=1.3, p_min=1, p_m
                   milestones=(), literal_phase=False, period_changes=(), lr_warmup_steps=0,
                   lr_warmup_len=1) -> Schedule:
     """period_changes: ((k, p), ...) for PIECEWISE: p from iteration k on.  lr_warmup_steps > 0: the
-    step size climbs lr0, 2 lr0, ... over that many stairs of lr_warmup_len iterations (Sec. V-C)."""
+    step size climbs lr0, 2 lr0, ... over that many stairs of lr_warmup_len iterations (Sec. IV-C)."""
     ms = (C.c_int64 * max(1, len(milestones)))(*milestones)
     pk = (C.c_int64 * max(1, len(period_changes)))(*[k for k, _ in period_changes])
     pv = (C.c_int32 * max(1, len(period_changes)))(*[p for _, p in period_changes])

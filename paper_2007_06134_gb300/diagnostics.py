@@ -1,6 +1,6 @@
 """Diagnostics of a run from its recorded trace (host-side, O(K)).
 
-The paper measures how far the replicas drift apart with Var[W_k] (Sec. III) and summarises a
+The paper measures how far the replicas drift apart with Var[W_k] (Sec. II-B) and summarises a
 schedule by the interval means V_t (Eq. vt) and the step-size-weighted mean variance (Eq.
 metric2), which bounds the convergence metric of Eq. metric1 (Eq. bound1).  With the trace
 option `var`, adpsgd_run records Var[W_k] at the start of every iteration k; these functions

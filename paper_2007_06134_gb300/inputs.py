@@ -3,7 +3,7 @@
 This module holds none of the method's arithmetic: it only draws the data the
 method runs on, from numpy's PCG64 generator with a stated seed.  The data
 stand in for the paper's image-classification workloads (CIFAR-10 / ImageNet
-CNN training, Sec. V), which are not available: every replica holds a flat
+CNN training, Sec. IV), which are not available: every replica holds a flat
 fp32 parameter vector sized like a CNN, and the objective is the separable
 quadratic f(x) = 1/2 sum_j h_j (x_j - c_j)^2, whose curvatures h_j and minimiser
 c_j are drawn here.
@@ -32,8 +32,8 @@ class Workload:
     lr0: float             # initial step size
     milestones: tuple = () # iterations where the step size is multiplied by lr_factor
     lr_factor: float = 0.1
-    p_init: int = 4        # Algorithm 2's p_init (Sec. V-B uses 4)
-    K_s_frac: float = 0.25 # K_s = K_s_frac * K (Sec. V-B uses 0.25K)
+    p_init: int = 4        # Algorithm 2's p_init (Sec. IV-B uses 4)
+    K_s_frac: float = 0.25 # K_s = K_s_frac * K (Sec. IV-B uses 0.25K)
     cpsgd_p: int = 8       # the comparison constant period
     noise: str = "philox"  # "philox" (fresh per step) or "bf16" (pre-materialised tensor)
     seed: int = DEFAULT_SEED
@@ -60,8 +60,8 @@ WORKLOADS = {
                          5e-4, 0.05),
 }
 
-# The schedule study of Sec. IV: 16 replicas, 4000 iterations, step size 0.1 x0.1 at 50 % and 75 %
-# of the run (the GoogLeNet / CIFAR-10 schedule of Sec. IV-A on a 2^20-parameter surrogate).
+# The schedule study of Sec. III: 16 replicas, 4000 iterations, step size 0.1 x0.1 at 50 % and 75 %
+# of the run (the GoogLeNet / CIFAR-10 schedule of Sec. III-A on a 2^20-parameter surrogate).
 WORKLOADS["strategies-n16"] = Workload("strategies-n16", 16, 1 << 20, 4000, "uniform:0.01:1", 1.0, 1.0, 0.9,
                                        5e-4, 0.1, milestones=(2000, 3000), K_s_frac=0.25)
 

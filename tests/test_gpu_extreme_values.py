@@ -3,7 +3,7 @@
 The kernels square deviations and loss terms in fp32 and add them in fp64; the oracle squares in
 fp64.  The two agree within 1e-4 as long as no fp32 square underflows or overflows.  Replicas that
 differ by less than about 2^-63 (subnormal parameters) or by more than about 2^63 break that.  For
-such columns the kernels redo the column in fp64, so the results follow the definition (Sec. III,
+such columns the kernels redo the column in fp64, so the results follow the definition (Sec. II-B,
 Var[W_k]) over the whole fp32 range.  These cases pin that:
 - tiny and huge values;
 - identical replicas and negative zeros;

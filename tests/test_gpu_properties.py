@@ -2,7 +2,7 @@
 plus randomised shapes against the oracle.
 
 - The spread of the replicas after m noisy steps from a common start has the exact second moment
-  of the linear recurrence (Sec. III's Var[W_k], statistical at 5 sigma): this pins the noise
+  of the linear recurrence (Sec. II-B's Var[W_k], statistical at 5 sigma): this pins the noise
   scale, the momentum form and D = sum_i ||x_i - xbar||^2 on the GPU without the oracle.
 - Averaging preserves the replica mean and leaves zero variance at P = 2^26.
 """

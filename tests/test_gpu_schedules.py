@@ -1,8 +1,8 @@
 """Schedule variants and the per-iteration variance record through the C ABI on the GPU.
 
-Piecewise-constant periods (the strategies of Sec. IV-A, the decreasing period of Sec. VI-B)
+Piecewise-constant periods (the strategies of Sec. III-A, the decreasing period of Sec. V-B)
 must sync where the oracle syncs (the paper's counts: 750, 750, 500) with bit-exact state, and
-the recorded Var[W_k] (Sec. III) must match the oracle's within 1e-4, exactly 0 after syncs."""
+the recorded Var[W_k] (Sec. II-B) must match the oracle's within 1e-4, exactly 0 after syncs."""
 import numpy as np
 import pytest
 
@@ -85,7 +85,7 @@ def test_variance_record_rejected_with_fused_intervals():
 
 
 def test_imagenet_style_schedule_run():
-    # Sec. V-C: step-size warm-up stairs, averaging every iteration during the warm-up (K_w), then
+    # Sec. IV-C: step-size warm-up stairs, averaging every iteration during the warm-up (K_w), then
     # Algorithm 2; the run must match the oracle bit for bit.
     w = inputs.WORKLOADS["quadratic-n4-P1M"]
     n, P, L = 4, 2053, 5

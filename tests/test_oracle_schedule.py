@@ -1,7 +1,7 @@
 """Pins of the oracle's schedules: Algorithm 1 (constant period) and Algorithm 2 (adaptive).
 
-Pinned by the sync-count arithmetic the paper prints (Sec. IV-A: 2000/4 + 2000/8
-= 750 and 4000/5 = 800; Sec. VI-B: 2000/20 + 2000/5 = 500 = 4000/8; Sec. IV-B:
+Pinned by the sync-count arithmetic the paper prints (Sec. III-A: 2000/4 + 2000/8
+= 750 and 4000/5 = 800; Sec. V-B: 2000/20 + 2000/5 = 500 = 4000/8; Sec. III-B:
 4000/498 ~ 8.03), by Algorithm 2's own logic on scripted variances (strict
 comparisons at 0.7 and 1.3, cumulative-mean C_2, p >= 1), and by closed forms of
 the noise-free run.
@@ -39,11 +39,11 @@ def test_literal_algorithm1_phase(K, p):
 
 def test_paper_sync_count_arithmetic():
     count = lambda K, p: O.schedule_only(cps(K, p), [])[0]
-    assert count(2000, 4) + count(2000, 8) == 750   # strategies 1 and 2 (Sec. IV-A)
+    assert count(2000, 4) + count(2000, 8) == 750   # strategies 1 and 2 (Sec. III-A)
     assert count(4000, 5) == 800                    # strategy 4
-    assert count(2000, 20) + count(2000, 5) == 500  # decreasing period of Sec. VI-B
+    assert count(2000, 20) + count(2000, 5) == 500  # decreasing period of Sec. V-B
     assert count(4000, 8) == 500
-    assert round(4000 / 498) == 8                   # equal-budget constant period (Sec. IV-B)
+    assert round(4000 / 498) == 8                   # equal-budget constant period (Sec. III-B)
 
 
 def test_adaptive_without_adaptation_is_constant_period():
@@ -211,7 +211,7 @@ def test_wire_bytes_ratios():
     K, P, n = 4000, 1000, 16
     full = O.wire_bytes(n, P, K, with_scalar=False)[0]
     adp = O.wire_bytes(n, P, K // 8, with_scalar=False)[0]
-    # 8-bit gradient quantisation moves 1/4 of full communication and twice ADPSGD (Sec. V-B).
+    # 8-bit gradient quantisation moves 1/4 of full communication and twice ADPSGD (Sec. IV-B).
     assert full / adp == pytest.approx(8.0) and (full / 4) / adp == pytest.approx(2.0)
 
 
@@ -242,8 +242,8 @@ def test_step_size_of_each_iteration_in_a_run():
 
 
 def test_piecewise_strategies_sync_counts():
-    # Sec. IV-A: strategy 1 (p = 4 for 2000 iterations, then 8) and strategy 2 (8, then 4) both
-    # sync 750 times in 4000 iterations; Sec. VI-B: 20 then 5 syncs 500 times.
+    # Sec. III-A: strategy 1 (p = 4 for 2000 iterations, then 8) and strategy 2 (8, then 4) both
+    # sync 750 times in 4000 iterations; Sec. V-B: 20 then 5 syncs 500 times.
     def count(p0, p1):
         spec = O.ScheduleSpec(kind=2, K=4000, p_init=p0, period_changes=((2000, p1),))
         return O.schedule_only(spec, [])
@@ -255,7 +255,7 @@ def test_piecewise_strategies_sync_counts():
 
 
 def test_variance_trace_resets_at_syncs_and_matches_second_moment():
-    # Var[W_k] (Sec. III) recorded at the start of every iteration: exactly 0 at k = 0 and right
+    # Var[W_k] (Sec. II-B) recorded at the start of every iteration: exactly 0 at k = 0 and right
     # after every sync, and t steps into an interval its mean is the second moment of the spread.
     n, P, p, K = 4, 1 << 14, 4, 40
     gamma, sigma = 0.1, 0.5
@@ -276,7 +276,7 @@ def test_variance_trace_resets_at_syncs_and_matches_second_moment():
 
 
 def test_imagenet_step_size_schedule():
-    # Sec. V-C: warm-up from 0.1, +0.1 per epoch for 8 epochs (0.8), x0.1 at epochs 30 and 60.
+    # Sec. IV-C: warm-up from 0.1, +0.1 per epoch for 8 epochs (0.8), x0.1 at epochs 30 and 60.
     L = 10  # iterations per epoch
     spec = O.ScheduleSpec(kind=0, K=90 * L, p_init=1, lr0=0.1, lr_factor=0.1, milestones=(30 * L, 60 * L),
                           lr_warmup_steps=8, lr_warmup_len=L)

@@ -1,12 +1,12 @@
 """Pins of the oracle's local step and its averaging + variance.
 
-Local step: Algorithm 1 / Algorithm 2 update line with SGD momentum (Sec. V-A)
+Local step: Algorithm 1 / Algorithm 2 update line with SGD momentum (Sec. IV-A)
 on the surrogate f(x) = 1/2 sum_j h_j (x_j - c_j)^2.  Pinned by closed forms of
 the linear recurrence (computed here by fp64 matrix powers, a different route
 from iterating), by the special case h = 0 where the update is a plain sum of
 the drawn noise, and by the exact second moment of the noise-driven spread.
 
-Averaging: Algorithm 2 averaging and S_k lines, Var[W_k] of Sec. III.  Pinned
+Averaging: Algorithm 2 averaging and S_k lines, Var[W_k] of Sec. II-B.  Pinned
 by n = 1 (identity), "variance is zero after each synchronization"
 (Sec. III-B), an exactly representable closed form, and fp64 brute force.
 """
@@ -137,7 +137,7 @@ def _noise_spread_expectation(h, gamma, sigma, mu, m, n):
 
 @pytest.mark.parametrize("mu", [0.0, 0.9])
 def test_variance_after_m_steps_matches_second_moment(mu):
-    # Statistical pin of the noise scale and of D = sum_i ||x_i - xbar||^2 (Sec. III).
+    # Statistical pin of the noise scale and of D = sum_i ||x_i - xbar||^2 (Sec. II-B).
     n, P, m, gamma, sigma = 4, 1 << 14, 6, 0.1, 0.5
     h, c = _problem(P)
     x = np.zeros((n, P), np.float32)
