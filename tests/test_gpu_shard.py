@@ -17,7 +17,13 @@ pytestmark = pytest.mark.gpu
 
 torch = pytest.importorskip("torch")
 DEV = "cuda:0"
-SUM_ORDER = 1e-12  # two fp64 summation orders of these sums differ by far less
+# S and the loss of a sharded run against the unsharded run.  With P % 4 == 0 every shard takes
+# the same float4 column groups as the unsharded run, whose fp32 group sums are then identical, and
+# only the order of the fp64 additions differs.  A ragged P runs the scalar kernels (one fp64 add
+# per column instead of one per fp32 group sum of four columns) where the shards' float4 kernels
+# differ from it by the fp32 rounding of those group sums, about 2^-24 relative.
+SUM_ORDER = 1e-12
+GROUP_ROUNDING = 1e-6
 
 
 def _dev(a):
@@ -104,15 +110,16 @@ def test_sharded_run_equals_unsharded_run(n, P, g, bf16, mode, track):
     sched = abi.make_schedule(abi.ADPSGD, K, 2, K_s=12, lr0=0.1, milestones=(30,))
     ux, uv, ut, ustats = _unsharded(n, P, sched, bf16=bf16, mode=mode, track=track, K=K)
     parts = _sharded(n, P, g, sched, bf16=bf16, mode=mode, track=track, K=K)
+    tol = SUM_ORDER if P % 4 == 0 else GROUP_ROUNDING
     for col0, cols, x, v, t, stats in parts:
         assert np.array_equal(x.view(np.uint32), ux[:, col0:col0 + cols].view(np.uint32)), col0
         assert np.array_equal(v.view(np.uint32), uv[:, col0:col0 + cols].view(np.uint32)), col0
         for key in ("k", "p", "phase"):
             assert np.array_equal(t[key], ut[key]), key
         for key in ("S", "loss", "C2"):
-            assert np.all(_rel(t[key], ut[key]) <= SUM_ORDER), key
+            assert np.all(_rel(t[key], ut[key]) <= tol), key
         if track:
-            assert np.all((_rel(t["var"][1:], ut["var"][1:]) <= SUM_ORDER))
+            assert np.all((_rel(t["var"][1:], ut["var"][1:]) <= tol))
         assert stats.rounds == ustats.rounds
         assert stats.wire_bytes_per_node == ustats.wire_bytes_per_node  # accounted on the whole P
     # every shard saw the same totals, bit for bit
