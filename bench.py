@@ -335,7 +335,7 @@ def run_gpu(args, w):
     noise = None
     if w.noise == "bf16":
         noise = torch.empty((n, P), dtype=torch.int16, device=device)
-        abi.adpsgd_noise_fill_bf16_shard(w.seed, n, P, col0, noise, stream)
+        abi.adpsgd_noise_fill_bf16_part(w.seed, n, P, 0, col0, noise, stream)
     fuse_sync = not args.no_sync_fusion
     noise_mode = abi.NOISE_BF16 if noise is not None else abi.NOISE_PHILOX
 

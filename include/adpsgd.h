@@ -288,15 +288,58 @@ typedef struct {
  * P_total < col0 + P, (col0 + P) / 4 >= 2^32, gather NULL with shards > 1). */
 int adpsgd_set_shard(adpsgd_ctx* ctx, const adpsgd_shard* shard);
 
+/* Replica split: the paper's own mapping (Sec. IV-A), one process per node holding whole
+ * replicas, averaging by an allreduce over the processes.  Process r holds cfg.n = n_local
+ * replicas, the global replicas [replica0, replica0 + n_local) (Philox counter word 1 is the
+ * global replica index), and owns one column chunk [col0, col0 + P_chunk) of the averaging.
+ *
+ * A sync runs as an allreduce split into its two halves, with the averaging kernel between them,
+ * so that the mean is the one of Algorithm 2 formed column by column over all n_total replicas in
+ * replica order (bit-identical to a single process holding them all):
+ *   1. collective(ADPSGD_SCATTER_COLUMNS, user): the caller's all-to-all, enqueued on the context's
+ *      stream, that leaves in chunk_x [n_total, P_chunk] every replica's values of this process's
+ *      chunk, in global replica order (reduce-scatter's traffic: (g - 1)/g of the parameters);
+ *   2. the averaging kernel on chunk_x (the chunk's mean, written to every row of chunk_x), its D
+ *      and loss over the chunk;
+ *   3. collective(ADPSGD_GATHER_AVERAGE, user): the caller's all-gather, enqueued on the stream,
+ *      of every chunk's mean (row 0 of each process's chunk_x) into every row of x;
+ *   4. the chunk sums through `gather`, added in process order (as for column shards).
+ * A collective returns 0, or nonzero for ADPSGD_E_PEER.  Every process calls them at the same
+ * syncs.  Not available with cfg.fuse_intervals, cfg.fuse_sync_step or the variance record. */
+enum { ADPSGD_SCATTER_COLUMNS = 0, ADPSGD_GATHER_AVERAGE = 1 };
+typedef int (*adpsgd_collective_fn)(int32_t op, void* user);
+
+typedef struct {
+    int32_t processes;       /* g >= 1 */
+    int32_t rank;            /* this process, 0 <= rank < processes */
+    int32_t replica0;        /* global index of this process's first replica */
+    int32_t n_total;         /* replicas of the whole problem (>= replica0 + cfg.n) */
+    int64_t col0;            /* this process's chunk of the averaging: columns [col0, col0 + P_chunk), */
+    int64_t P_chunk;         /* col0 a multiple of 4, col0 + P_chunk <= cfg.P */
+    float* chunk_x;          /* device [n_total, P_chunk], 16-byte aligned */
+    adpsgd_collective_fn collective;
+    adpsgd_gather_fn gather; /* every process's chunk sums, in process order (NULL with one process) */
+    void* user;              /* passed to collective and gather */
+} adpsgd_replica_split;
+
+/* Make ctx one process of a replica split (before its first step).  chunk_x and the chunk's
+ * slices of h and c (h + col0, c + col0) must stay valid until adpsgd_destroy.
+ * Errors: E_INVAL (ranges, NULL collective, gather NULL with processes > 1, fuse_intervals or
+ * fuse_sync_step set), E_ALIGN (chunk_x, or col0 leaving h + col0 unaligned). */
+int adpsgd_set_replica_split(adpsgd_ctx* ctx, const adpsgd_replica_split* split);
+
 /* The exchange alone, for tests and for callers that run their own averaging (pure host code):
  * gathers `count` doubles from every shard through shard->gather and writes their sums in shard
  * order, out[t] = ((0 + local_0[t]) + local_1[t]) + ...  Errors: E_INVAL, E_PEER. */
 int adpsgd_shard_combine(const adpsgd_shard* shard, const double* local, int64_t count, double* out);
 
-/* The bf16 noise tensor of one shard: columns [col0, col0 + P) of the [n, P_total] tensor that
- * adpsgd_noise_fill_bf16 fills, as an [n, P] array.  col0 a multiple of 4.  Enqueued only.
- * Errors: as adpsgd_noise_fill_bf16, and E_INVAL for col0. */
-int adpsgd_noise_fill_bf16_shard(uint64_t seed, int32_t n, int64_t P, int64_t col0, uint16_t* out, void* stream);
+/* A part of the bf16 noise tensor that adpsgd_noise_fill_bf16 fills: rows (replicas)
+ * [replica0, replica0 + n) and columns [col0, col0 + P) of the whole [n_total, P_total] tensor, as an
+ * [n, P] array -- a column shard's slice (replica0 = 0) or a process's replicas (adpsgd_replica_split).
+ * col0 a multiple of 4.  Enqueued only.  Errors: as adpsgd_noise_fill_bf16, and E_INVAL for a
+ * negative replica0 or col0 not a multiple of 4. */
+int adpsgd_noise_fill_bf16_part(uint64_t seed, int32_t n, int64_t P, int32_t replica0, int64_t col0, uint16_t* out,
+                                void* stream);
 
 /* The period rule alone (Algorithm 2, after the sync at iteration k; pure host code):
  * warm-up (k < K_w) and kind 0 leave the state unchanged; k < K_s: m += 1,

@@ -76,6 +76,17 @@ class KernelTiming(C.Structure):
 GATHER_FN = C.CFUNCTYPE(C.c_int, C.POINTER(C.c_double), C.c_int64, C.POINTER(C.c_double), C.c_void_p)
 
 
+SCATTER_COLUMNS, GATHER_AVERAGE = 0, 1
+# int collective(int32_t op, void* user)
+COLLECTIVE_FN = C.CFUNCTYPE(C.c_int, C.c_int32, C.c_void_p)
+
+
+class ReplicaSplit(C.Structure):
+    _fields_ = [("processes", C.c_int32), ("rank", C.c_int32), ("replica0", C.c_int32), ("n_total", C.c_int32),
+                ("col0", C.c_int64), ("P_chunk", C.c_int64), ("chunk_x", C.c_void_p),
+                ("collective", COLLECTIVE_FN), ("gather", GATHER_FN), ("user", C.c_void_p)]
+
+
 class Shard(C.Structure):
     _fields_ = [("shards", C.c_int32), ("index", C.c_int32), ("col0", C.c_int64), ("P_total", C.c_int64),
                 ("gather", GATHER_FN), ("user", C.c_void_p)]
@@ -101,8 +112,9 @@ _SIGS = {
     "adpsgd_noise_fill_f32": (C.c_int, [C.c_uint64, C.c_uint32, C.c_int32, C.c_int64, C.c_int64, _P, _P]),
     "adpsgd_noise_fill_bf16": (C.c_int, [C.c_uint64, C.c_int32, C.c_int64, _P, _P]),
     "adpsgd_set_shard": (C.c_int, [_P, C.POINTER(Shard)]),
+    "adpsgd_set_replica_split": (C.c_int, [_P, C.POINTER(ReplicaSplit)]),
     "adpsgd_shard_combine": (C.c_int, [C.POINTER(Shard), C.POINTER(C.c_double), C.c_int64, C.POINTER(C.c_double)]),
-    "adpsgd_noise_fill_bf16_shard": (C.c_int, [C.c_uint64, C.c_int32, C.c_int64, C.c_int64, _P, _P]),
+    "adpsgd_noise_fill_bf16_part": (C.c_int, [C.c_uint64, C.c_int32, C.c_int64, C.c_int32, C.c_int64, _P, _P]),
     "adpsgd_copy_h2d": (C.c_int, [_P, _P, C.c_int64, _P]),
     "adpsgd_copy_d2h": (C.c_int, [_P, _P, C.c_int64, _P]),
     "adpsgd_kernel_times": (C.c_int, [_P, C.POINTER(KernelTiming)]),
@@ -241,6 +253,20 @@ def adpsgd_set_shard(ctx: Context, shard: Shard) -> None:
     ctx._shard = shard  # the context calls shard.gather until it is destroyed
 
 
+def make_replica_split(processes: int, rank: int, replica0: int, n_total: int, col0: int, P_chunk: int, chunk_x,
+                       collective, gather=None) -> ReplicaSplit:
+    """collective: a COLLECTIVE_FN; gather: a GATHER_FN (None with one process)."""
+    rs = ReplicaSplit(processes, rank, replica0, n_total, col0, P_chunk, _ptr(chunk_x), collective,
+                      gather if gather is not None else GATHER_FN(), None)
+    rs._keep = (chunk_x, collective, gather)
+    return rs
+
+
+def adpsgd_set_replica_split(ctx: Context, split: ReplicaSplit) -> None:
+    _check(load().adpsgd_set_replica_split(ctx.handle, C.byref(split)), "adpsgd_set_replica_split")
+    ctx._split = split  # the context calls split.collective and split.gather until it is destroyed
+
+
 def adpsgd_shard_combine(shard: Shard, local):
     """Every shard's values through shard.gather, summed in shard order (pure host code)."""
     import numpy as np
@@ -364,9 +390,10 @@ def adpsgd_noise_fill_bf16(seed: int, n: int, P: int, out, stream=None) -> None:
            "adpsgd_noise_fill_bf16")
 
 
-def adpsgd_noise_fill_bf16_shard(seed: int, n: int, P: int, col0: int, out, stream=None) -> None:
-    _check(load().adpsgd_noise_fill_bf16_shard(seed & 0xFFFFFFFFFFFFFFFF, n, P, col0, _ptr(out), _stream(stream)),
-           "adpsgd_noise_fill_bf16_shard")
+def adpsgd_noise_fill_bf16_part(seed: int, n: int, P: int, replica0: int, col0: int, out, stream=None) -> None:
+    """Rows [replica0, replica0 + n) and columns [col0, col0 + P) of the bf16 noise tensor."""
+    _check(load().adpsgd_noise_fill_bf16_part(seed & 0xFFFFFFFFFFFFFFFF, n, P, replica0, col0, _ptr(out),
+                                              _stream(stream)), "adpsgd_noise_fill_bf16_part")
 
 
 def _nbytes(t, nbytes):

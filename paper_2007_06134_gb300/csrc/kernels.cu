@@ -62,6 +62,7 @@ struct StepParams {
     int32_t n;
     uint32_t k;
     uint32_t q0;  // Philox block of the first column: the column offset of a shard, divided by 4
+    uint32_t r0;  // global index of replica 0 (the first replica of a replica split)
     float gamma, mu, wd, sigma;
     PhiloxKeys keys;
 };
@@ -103,7 +104,7 @@ __global__ void __launch_bounds__(kStepThreads) local_step_kernel(const StepPara
         for (int g = 0; g < kStepGroups; ++g) {
             const int64_t q = q0 + g * kStepThreads;
             if (q >= p.Q) break;
-            const float4 z = BF16 ? zb[g] : normals4(p.keys, (uint32_t)q + p.q0, (uint32_t)i, p.k, 0u);
+            const float4 z = BF16 ? zb[g] : normals4(p.keys, (uint32_t)q + p.q0, (uint32_t)i + p.r0, p.k, 0u);
             sgd_update<WD>(xv[g].x, vv[g].x, hv[g].x, cv[g].x, z.x, p.gamma, p.mu, p.wd, p.sigma);
             sgd_update<WD>(xv[g].y, vv[g].y, hv[g].y, cv[g].y, z.y, p.gamma, p.mu, p.wd, p.sigma);
             sgd_update<WD>(xv[g].z, vv[g].z, hv[g].z, cv[g].z, z.z, p.gamma, p.mu, p.wd, p.sigma);
@@ -117,7 +118,7 @@ __global__ void __launch_bounds__(kStepThreads) local_step_kernel(const StepPara
             if (q >= p.Q) break;
             float zz[4];
             if (!BF16) {
-                const float4 z = normals4(p.keys, (uint32_t)q + p.q0, (uint32_t)i, p.k, 0u);
+                const float4 z = normals4(p.keys, (uint32_t)q + p.q0, (uint32_t)i + p.r0, p.k, 0u);
                 zz[0] = z.x; zz[1] = z.y; zz[2] = z.z; zz[3] = z.w;
             }
 #pragma unroll
@@ -220,12 +221,12 @@ __global__ void __launch_bounds__(kThreads) noise_f32_kernel(PhiloxKeys keys, ui
 }
 
 __global__ void __launch_bounds__(kThreads) noise_bf16_kernel(PhiloxKeys keys, int32_t n, int64_t P,
-                                                              int64_t Q, uint32_t q0, uint16_t* out)
+                                                              int64_t Q, uint32_t r0, uint32_t q0, uint16_t* out)
 {
     const int64_t t = (int64_t)blockIdx.x * kThreads + threadIdx.x;
     if (t >= (int64_t)n * Q) return;
     const int64_t i = t / Q, q = t % Q;
-    const float4 z = normals4(keys, (uint32_t)q + q0, (uint32_t)i, 0u, 1u);
+    const float4 z = normals4(keys, (uint32_t)q + q0, (uint32_t)i + r0, 0u, 1u);
     const float zz[4] = {z.x, z.y, z.z, z.w};
 #pragma unroll
     for (int r = 0; r < 4; ++r)
@@ -295,6 +296,7 @@ cudaError_t launch_local_step(const LocalStepArgs& a, cudaStream_t stream)
     p.n = a.n;
     p.k = a.k;
     p.q0 = a.q0;
+    p.r0 = a.r0;
     p.gamma = a.gamma;
     p.mu = a.mu;
     p.wd = a.wd;
@@ -374,14 +376,15 @@ cudaError_t launch_noise_f32(uint64_t seed, uint32_t tag, int32_t n, int64_t P, 
     return cudaGetLastError();
 }
 
-cudaError_t launch_noise_bf16(uint64_t seed, int32_t n, int64_t P, uint32_t q0, uint16_t* out, cudaStream_t stream)
+cudaError_t launch_noise_bf16(uint64_t seed, int32_t n, int64_t P, uint32_t r0, uint32_t q0, uint16_t* out,
+                              cudaStream_t stream)
 {
     PhiloxKeys keys;
     make_philox_keys(seed, &keys);
     const int64_t Q = ceil_div(P, 4);
     const int64_t blocks = ceil_div((int64_t)n * Q, kThreads);
     if (blocks == 0) return cudaSuccess;
-    noise_bf16_kernel<<<(unsigned)blocks, kThreads, 0, stream>>>(keys, n, P, Q, q0, out);
+    noise_bf16_kernel<<<(unsigned)blocks, kThreads, 0, stream>>>(keys, n, P, Q, r0, q0, out);
     return cudaGetLastError();
 }
 

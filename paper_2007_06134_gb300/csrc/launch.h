@@ -29,6 +29,7 @@ struct LocalStepArgs {
     int64_t P;
     uint32_t k;
     uint32_t q0;  // Philox block of column 0 (a shard's column offset / 4; 0 unsharded)
+    uint32_t r0;  // global index of replica 0 (a replica split's first replica; 0 otherwise)
     float gamma, mu, wd, sigma;
 };
 cudaError_t launch_local_step(const LocalStepArgs& a, cudaStream_t stream);
@@ -122,8 +123,8 @@ cudaError_t launch_philox_fill(uint64_t seed, uint32_t tag, int32_t n, int64_t n
                                uint32_t* out, cudaStream_t stream);
 cudaError_t launch_noise_f32(uint64_t seed, uint32_t tag, int32_t n, int64_t P, uint32_t k,
                              float* out, cudaStream_t stream);
-// The bf16 noise tensor of columns [4 q0, 4 q0 + P) of the whole problem.
-cudaError_t launch_noise_bf16(uint64_t seed, int32_t n, int64_t P, uint32_t q0, uint16_t* out,
+// Rows [r0, r0 + n) and columns [4 q0, 4 q0 + P) of the bf16 noise tensor of the whole problem.
+cudaError_t launch_noise_bf16(uint64_t seed, int32_t n, int64_t P, uint32_t r0, uint32_t q0, uint16_t* out,
                               cudaStream_t stream);
 
 }  // namespace adpsgd

@@ -102,10 +102,18 @@ struct adpsgd_ctx {
     int64_t launches[4] = {0, 0, 0, 0};
     int64_t timed_launches[4] = {0, 0, 0, 0};
     bool force_incomplete = false;
-    // column sharding (adpsgd_set_shard): the Philox block of column 0 and the exchange
+    // column sharding (adpsgd_set_shard): the Philox block of column 0 and the exchange of the
+    // partial sums (also used by a replica split)
     uint32_t q0 = 0;
     bool sharded = false;
     adpsgd_shard shard{};
+    // replica split (adpsgd_set_replica_split): this process's first global replica, the
+    // replicas of the whole problem, the averaging's column chunk and its grids
+    bool replica = false;
+    adpsgd_replica_split split{};
+    uint32_t r0 = 0;
+    int32_t n_total = 0;  // replicas of the whole problem (cfg.n unless split)
+    int grid_chunk = 0, grid_chunk_loss = 0, grid_chunk_var = 0;
 };
 
 namespace {
@@ -222,6 +230,7 @@ int local_step(adpsgd_ctx* ctx, int64_t k, float gamma)
     a.P = ctx->cfg.P;
     a.k = (uint32_t)k;
     a.q0 = ctx->q0;
+    a.r0 = ctx->r0;
     a.gamma = gamma;
     a.mu = ctx->cfg.momentum;
     a.wd = ctx->cfg.weight_decay;
@@ -229,10 +238,45 @@ int local_step(adpsgd_ctx* ctx, int64_t k, float gamma)
     return timed(ctx, 0, [&] { return adpsgd::launch_local_step(a, ctx->stream); }, "local step");
 }
 
+// A replica split's sync: the caller's all-to-all into the chunk, the averaging (or variance)
+// kernel on the chunk of all replicas, the copy of its two sums into ctx->h_out and ctx->done, and
+// (write_back) the caller's all-gather of the chunks' means into x.
+int replica_average_enqueue(adpsgd_ctx* ctx, bool write_back, bool loss)
+{
+    const adpsgd_replica_split& rs = ctx->split;
+    if (rs.collective(ADPSGD_SCATTER_COLUMNS, rs.user) != 0) {
+        g_last_error = "the replica split's all-to-all failed";
+        return ADPSGD_E_PEER;
+    }
+    adpsgd::AverageArgs a;
+    a.x = rs.chunk_x;
+    a.h = loss ? ctx->h + rs.col0 : nullptr;
+    a.c = loss ? ctx->c + rs.col0 : nullptr;
+    a.n = rs.n_total;
+    a.P = rs.P_chunk;
+    a.write_back = write_back;
+    a.partials = ctx->d_partials;
+    a.out = ctx->d_out;
+    a.counter = reinterpret_cast<unsigned int*>(ctx->d_out + 2);
+    a.grid = !write_back ? ctx->grid_chunk_var : (loss ? ctx->grid_chunk_loss : ctx->grid_chunk);
+    int st = timed(ctx, 1, [&] { return adpsgd::launch_average(a, ctx->stream); }, "average");
+    if (st != ADPSGD_OK) return st;
+    cudaError_t e = cudaMemcpyAsync(ctx->h_out, ctx->d_out, 2 * sizeof(double), cudaMemcpyDeviceToHost,
+                                    ctx->stream);
+    if (e == cudaSuccess) e = cudaEventRecord(ctx->done, ctx->stream);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaMemcpyAsync");
+    if (write_back && rs.collective(ADPSGD_GATHER_AVERAGE, rs.user) != 0) {
+        g_last_error = "the replica split's all-gather failed";
+        return ADPSGD_E_PEER;
+    }
+    return ADPSGD_OK;
+}
+
 // Enqueue the averaging (write_back) or variance-only kernel and the copy of its two sums
 // into ctx->h_out, then record ctx->done.
 int average_enqueue(adpsgd_ctx* ctx, bool write_back, bool loss)
 {
+    if (ctx->replica) return replica_average_enqueue(ctx, write_back, loss);
     adpsgd::AverageArgs a;
     a.x = ctx->x;
     a.h = loss ? ctx->h : nullptr;
@@ -501,6 +545,7 @@ int adpsgd_init(const adpsgd_config* cfg, float* x, float* v, const float* h, co
     ctx->c = c;
     ctx->noise = cfg->noise_mode == ADPSGD_NOISE_BF16 ? noise_bf16 : nullptr;
     ctx->stream = static_cast<cudaStream_t>(stream);
+    ctx->n_total = cfg->n;
     adpsgd::make_philox_keys(cfg->seed, &ctx->keys);
 
     cudaError_t e = cudaGetDevice(&ctx->device);
@@ -651,7 +696,7 @@ int adpsgd_run(adpsgd_ctx* ctx, const adpsgd_schedule* sched, adpsgd_state* stat
     const bool loss = ctx->cfg.want_loss != 0;
     const int64_t stop = k_end < sched->K ? k_end : sched->K;
     const bool track = trace != nullptr && trace->var != nullptr && trace->var_cap > 0;
-    if (track && ctx->cfg.fuse_intervals) return ADPSGD_E_INVAL;
+    if (track && (ctx->cfg.fuse_intervals || ctx->replica)) return ADPSGD_E_INVAL;
     if (track && stop > ctx->d_var_cap) {
         if (ctx->d_var != nullptr) {
             cudaError_t e = cudaStreamSynchronize(ctx->stream);
@@ -707,7 +752,7 @@ int adpsgd_run(adpsgd_ctx* ctx, const adpsgd_schedule* sched, adpsgd_state* stat
                 st = sync_sums(ctx, &D, &L);
                 if (st != ADPSGD_OK) return st;
                 const int64_t ks = k + m - 1;
-                const double S = D / (double)ctx->cfg.n;
+                const double S = D / (double)ctx->n_total;
                 const int32_t phase = rule(sched, state, ks, S, (double)gam[m - 1]);
                 if (trace != nullptr && trace->len < trace->cap) {
                     const int64_t t = trace->len;
@@ -761,7 +806,7 @@ int adpsgd_run(adpsgd_ctx* ctx, const adpsgd_schedule* sched, adpsgd_state* stat
         double D = 0.0, L = 0.0;
         st = sync_sums(ctx, &D, &L);
         if (st != ADPSGD_OK) return st;
-        const double S = D / (double)ctx->cfg.n;
+        const double S = D / (double)ctx->n_total;
         const int32_t phase = rule(sched, state, k, S, (double)gamma_of(sched, k));
         if (trace != nullptr) {
             if (trace->len < trace->cap) {
@@ -794,7 +839,7 @@ int adpsgd_run(adpsgd_ctx* ctx, const adpsgd_schedule* sched, adpsgd_state* stat
                 st = shard_combine(&ctx->shard, local.data(), (int64_t)local.size(), D.data());
                 if (st != ADPSGD_OK) return st;
             }
-            for (int64_t k = k_first; k < last; ++k) trace->var[k] = D[(size_t)(k - k_first)] / (double)ctx->cfg.n;
+            for (int64_t k = k_first; k < last; ++k) trace->var[k] = D[(size_t)(k - k_first)] / (double)ctx->n_total;
         }
     }
     if (stats != nullptr) {
@@ -802,8 +847,8 @@ int adpsgd_run(adpsgd_ctx* ctx, const adpsgd_schedule* sched, adpsgd_state* stat
         stats->equiv_period = state->rounds > 0 ? (double)state->k_next / (double)state->rounds : 0.0;
         double total = 0.0;
         const int64_t P_all = ctx->sharded ? ctx->shard.P_total : ctx->cfg.P;
-        wire(ctx->cfg.n, P_all, state->rounds, true, &stats->wire_bytes_per_node, &stats->wire_bytes_total);
-        wire(ctx->cfg.n, P_all, state->k_next, false, &stats->fullsgd_wire_bytes_per_node, &total);
+        wire(ctx->n_total, P_all, state->rounds, true, &stats->wire_bytes_per_node, &stats->wire_bytes_total);
+        wire(ctx->n_total, P_all, state->k_next, false, &stats->fullsgd_wire_bytes_per_node, &total);
         stats->local_step_launches = ctx->launches[0] - launches0[0];
         stats->average_launches = ctx->launches[1] - launches0[1];
         stats->interval_launches = ctx->launches[2] - launches0[2];
@@ -892,28 +937,53 @@ int adpsgd_noise_fill_bf16(uint64_t seed, int32_t n, int64_t P, uint16_t* out, v
     if (out == nullptr || n < 0 || P < 0 || P > (int64_t(1) << 34)) return ADPSGD_E_INVAL;
     if ((int64_t)n * P > (int64_t(1) << 40)) return ADPSGD_E_INVAL;
     if (!aligned16(out)) return ADPSGD_E_ALIGN;
-    cudaError_t e = adpsgd::launch_noise_bf16(seed, n, P, 0u, out, static_cast<cudaStream_t>(stream));
+    cudaError_t e = adpsgd::launch_noise_bf16(seed, n, P, 0u, 0u, out, static_cast<cudaStream_t>(stream));
     return e == cudaSuccess ? ADPSGD_OK : cuda_fail(e, "bf16 noise fill");
 }
 
-int adpsgd_noise_fill_bf16_shard(uint64_t seed, int32_t n, int64_t P, int64_t col0, uint16_t* out, void* stream)
+int adpsgd_noise_fill_bf16_part(uint64_t seed, int32_t n, int64_t P, int32_t replica0, int64_t col0, uint16_t* out,
+                                void* stream)
 {
-    if (out == nullptr || n < 0 || P < 0 || P > (int64_t(1) << 34)) return ADPSGD_E_INVAL;
+    if (out == nullptr || n < 0 || P < 0 || P > (int64_t(1) << 34) || replica0 < 0) return ADPSGD_E_INVAL;
     if (col0 < 0 || col0 % 4 != 0 || (col0 + P + 3) / 4 > kMaxK) return ADPSGD_E_INVAL;
     if ((int64_t)n * P > (int64_t(1) << 40)) return ADPSGD_E_INVAL;
     if (!aligned16(out)) return ADPSGD_E_ALIGN;
-    cudaError_t e = adpsgd::launch_noise_bf16(seed, n, P, (uint32_t)(col0 / 4), out, static_cast<cudaStream_t>(stream));
+    cudaError_t e = adpsgd::launch_noise_bf16(seed, n, P, (uint32_t)replica0, (uint32_t)(col0 / 4), out,
+                                              static_cast<cudaStream_t>(stream));
     return e == cudaSuccess ? ADPSGD_OK : cuda_fail(e, "bf16 noise fill");
 }
 
 int adpsgd_set_shard(adpsgd_ctx* ctx, const adpsgd_shard* shard)
 {
-    if (ctx == nullptr || check_shard(shard) != ADPSGD_OK) return ADPSGD_E_INVAL;
+    if (ctx == nullptr || ctx->replica || check_shard(shard) != ADPSGD_OK) return ADPSGD_E_INVAL;
     if (shard->P_total < shard->col0 + ctx->cfg.P) return ADPSGD_E_INVAL;
     if ((shard->col0 + ctx->cfg.P + 3) / 4 > kMaxK) return ADPSGD_E_INVAL;  // Philox blocks are 32-bit words
     ctx->shard = *shard;
     ctx->sharded = true;
     ctx->q0 = (uint32_t)(shard->col0 / 4);
+    return ADPSGD_OK;
+}
+
+int adpsgd_set_replica_split(adpsgd_ctx* ctx, const adpsgd_replica_split* rs)
+{
+    if (ctx == nullptr || rs == nullptr || ctx->sharded) return ADPSGD_E_INVAL;
+    if (rs->processes < 1 || rs->rank < 0 || rs->rank >= rs->processes || rs->collective == nullptr) return ADPSGD_E_INVAL;
+    if (rs->processes > 1 && rs->gather == nullptr) return ADPSGD_E_INVAL;
+    if (rs->replica0 < 0 || rs->n_total < 1 || (int64_t)rs->replica0 + ctx->cfg.n > rs->n_total) return ADPSGD_E_INVAL;
+    if (rs->col0 < 0 || rs->col0 % 4 != 0 || rs->P_chunk < 0 || rs->col0 + rs->P_chunk > ctx->cfg.P) return ADPSGD_E_INVAL;
+    if ((int64_t)rs->n_total * rs->P_chunk > (int64_t(1) << 40)) return ADPSGD_E_INVAL;
+    if (rs->chunk_x == nullptr || ctx->cfg.fuse_intervals || ctx->cfg.fuse_sync_step) return ADPSGD_E_INVAL;
+    if (!aligned16(rs->chunk_x) || !aligned16(ctx->h + rs->col0) || !aligned16(ctx->c + rs->col0)) return ADPSGD_E_ALIGN;
+    ctx->split = *rs;
+    ctx->replica = true;
+    ctx->r0 = (uint32_t)rs->replica0;
+    ctx->n_total = rs->n_total;
+    ctx->grid_chunk = adpsgd::average_grid(rs->n_total, rs->P_chunk, false, true, ctx->sms);
+    ctx->grid_chunk_loss = adpsgd::average_grid(rs->n_total, rs->P_chunk, true, true, ctx->sms);
+    ctx->grid_chunk_var = adpsgd::average_grid(rs->n_total, rs->P_chunk, false, false, ctx->sms);
+    // the chunk sums are exchanged like a column shard's (process order); x keeps every column
+    ctx->shard = adpsgd_shard{rs->processes, rs->rank, 0, ctx->cfg.P, rs->gather, rs->user};
+    ctx->sharded = true;
     return ADPSGD_OK;
 }
 

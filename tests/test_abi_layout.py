@@ -26,6 +26,7 @@ STRUCTS = {
     "adpsgd_stats": abi.Stats,
     "adpsgd_kernel_timing": abi.KernelTiming,
     "adpsgd_shard": abi.Shard,
+    "adpsgd_replica_split": abi.ReplicaSplit,
 }
 
 

@@ -74,7 +74,7 @@ def _sharded(n, P, g, sched, *, bf16, mode, track, K):
                 nd = None
                 if bf16:
                     nd = torch.empty((n, cols), dtype=torch.int16, device=DEV)
-                    abi.adpsgd_noise_fill_bf16_shard(seed, n, cols, col0, nd, stream)
+                    abi.adpsgd_noise_fill_bf16_part(seed, n, cols, 0, col0, nd, stream)
             stream.synchronize()
             tr = abi.TraceBuffers(K + 1, var_cap=K if track else 0)
             with abi.adpsgd_init(_cfg(n, cols, bf16=bf16, mode=mode, seed=seed), xd, vd, hd, cd, nd, stream) as ctx:

@@ -118,3 +118,53 @@ def test_combine_between_two_gloo_processes():
     got = dict(q.get(timeout=10) for _ in range(2))
     want = [(0.0 + 1e16) + 1.0, (0.0 + 0.1) + 0.2, (0.0 + -0.0) + -3.0]
     assert got[0] == got[1] == want
+
+
+def _replica_worker(rank, world, port, q):
+    os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port), RANK=str(rank), WORLD_SIZE=str(world))
+    sys.path.insert(0, ROOT)
+    import torch
+    import torch.distributed as dist
+
+    from paper_2007_06134_gb300 import abi as A
+    from paper_2007_06134_gb300 import shard as S
+    dist.init_process_group("gloo", rank=rank, world_size=world)
+    n_locals = [2, 1]
+    P = 4 * 5 + 3
+    x = torch.arange(n_locals[rank] * P, dtype=torch.float32).reshape(n_locals[rank], P) + 1000.0 * rank
+    c0, cols = S.column_split(P, world, rank)
+    chunk = torch.full((sum(n_locals), cols), -1.0)
+    coll = S.DistReplicaCollective(x, chunk, n_locals)
+    assert coll.callback(A.SCATTER_COLUMNS, None) == 0
+    scattered = chunk.clone()
+    chunk[0] = 0.5 + rank + torch.arange(cols, dtype=torch.float32)  # stands in for the chunk's mean
+    assert coll.callback(A.GATHER_AVERAGE, None) == 0
+    q.put((rank, scattered.tolist(), x.tolist()))
+    dist.destroy_process_group()
+
+
+def test_replica_split_collectives_between_two_gloo_processes():
+    # The all-to-all leaves every process all replicas' values of its column chunk, rows in global
+    # replica order (process 0's two replicas, then process 1's); the all-gather writes every
+    # chunk's row 0 into every local replica.
+    import torch.multiprocessing as mp
+    ctx = mp.get_context("spawn")
+    q = ctx.Queue()
+    port = _free_port()
+    procs = [ctx.Process(target=_replica_worker, args=(r, 2, port, q)) for r in range(2)]
+    for p in procs:
+        p.start()
+    for p in procs:
+        p.join(180)
+        assert p.exitcode == 0
+    got = dict((r, (np.array(a), np.array(b))) for r, a, b in (q.get(timeout=10) for _ in range(2)))
+    P = 23
+    x_all = np.concatenate([np.arange(2 * P, dtype=np.float32).reshape(2, P),
+                            np.arange(P, dtype=np.float32).reshape(1, P) + 1000.0])
+    mean_row = np.concatenate([0.5 + r + np.arange(shard.column_split(P, 2, r)[1], dtype=np.float32)
+                               for r in range(2)])
+    for r in range(2):
+        c0, cols = shard.column_split(P, 2, r)
+        scattered, x_after = got[r]
+        assert np.array_equal(scattered, x_all[:, c0:c0 + cols])
+        assert np.array_equal(x_after, np.repeat(mean_row[None, :], x_after.shape[0], axis=0))
