@@ -30,14 +30,24 @@ struct SyncStepParams {
 };
 
 // Register cap: 128 per thread (2 blocks of 256 per SM) up to 8 replicas, 255 for 16.  One
-// thread per column group.  Other forms measured slower on resnet18-n8 (0.316 ms here):
+// thread per column group.  Other forms measured slower on resnet18-n8 (0.314 ms here, one launch
+// under ncu; 225 M warp-instructions at 60 % issue):
 // - splitting a group's replicas over two lanes that swap halves by shuffles (0.346 ms);
 // - a tiled form, with a thread per (group, replica) as in local_step_kernel and the averaging
 //   from a shared-memory tile (0.350 ms);
 // - the step over the replicas in chunks of 4 under a runtime loop, stashing the new x in shared
 //   memory, to shrink the unrolled code (0.336 ms);
 // - this form capped at 80 registers for 3 blocks per SM, which spills (0.426 ms);
-// - 128-thread blocks at 96 registers, 5 per SM, no spills (0.337 ms).
+// - 128-thread blocks at 96 registers, 5 per SM, no spills (0.337 ms);
+// - loads streamed through shared memory by per-thread cp.async copies, refilled replica by
+//   replica for the next group, 6 blocks of 128 per SM: 0.333 ms with the replicas unrolled
+//   (250 M instructions, instruction-fetch stalls 2.0 per issue), 0.314 ms with a replica loop
+//   that is not unrolled (258 M instructions at 72 % issue: the copies' per-thread address work
+//   takes what the higher issue rate gains);
+// - a tile per block with a barrier, each thread stepping two (replica, group) items and then
+//   averaging whole columns of the tile: 0.469 ms (400 M instructions);
+// - per-warp bulk copies (cp.async.bulk on mbarriers, lane 0 refilling a 3-stage ring): 0.396 ms
+//   (351 M instructions, most of the excess in the waits).
 template <int NMAX, bool BF16, bool LOSS>
 __global__ void __launch_bounds__(kThreads, (NMAX >= 16 ? 1 : 2)) sync_step_kernel(const SyncStepParams p)
 {
@@ -89,113 +99,6 @@ __global__ void __launch_bounds__(kThreads, (NMAX >= 16 ? 1 : 2)) sync_step_kern
     finish_sums<LOSS>(a, accD, accL);
 }
 
-// ------------------------------------------------------------------------------------------
-// Pipelined form (Philox noise, 3..16 replicas): the loads go through shared memory by
-// per-thread asynchronous copies (cp.async), so data in flight holds no registers.
-// ------------------------------------------------------------------------------------------
-// Each thread owns one float4 column group of all n replicas per iteration of a persistent
-// grid-stride loop, as in sync_step_kernel.  Its shared-memory slots hold x_i and v_i of every
-// replica i (and h, c), slot-major with the block's threads consecutive (conflict-free 16-byte
-// accesses).  One commit group per replica: the copies of (group q, replica i) are waited for
-// just before replica i is stepped, and as soon as it has been read its slots are refilled with
-// (next group, replica i).  So while a thread steps the rest of group q and averages it, the
-// copies for the next group are in flight: up to n * 32 bytes per thread without holding a
-// register, on more resident warps than the register-resident form (whose loads held 2 n float4).
-// The arithmetic is the local step's and the averaging's, in the same order (bit-identical).
-constexpr int kPipeThreads = 128;
-
-__device__ __forceinline__ void cp_async16(float4* smem_dst, const float4* gmem_src)
-{
-    const unsigned dst = (unsigned)__cvta_generic_to_shared(smem_dst);
-    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;\n" ::"r"(dst), "l"(gmem_src) : "memory");
-}
-
-__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;\n" ::: "memory"); }
-
-// Wait until at most N of this thread's most recent commit groups are still in flight.
-template <int N>
-__device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;\n" ::"n"(N) : "memory"); }
-
-template <int NMAX>
-constexpr int pipe_slots() { return 2 * NMAX + 2; }  // x_i, v_i per replica, then h and c
-
-// Issue the copies of (group q, replica i) into the thread's slots; h and c ride with replica 0.
-// Out-of-range groups and inactive replicas issue nothing (their commit group stays empty).
-template <int NMAX>
-__device__ __forceinline__ void pipe_fill(const SyncStepParams& p, float4* slots, int64_t q, int i)
-{
-    const AvgParams& a = p.avg;
-    if (q >= a.Q || i >= a.n) return;
-    const int64_t row = (int64_t)i * a.P;
-    cp_async16(slots + (2 * i) * kPipeThreads, reinterpret_cast<const float4*>(a.x + row) + q);
-    cp_async16(slots + (2 * i + 1) * kPipeThreads, reinterpret_cast<const float4*>(p.v + row) + q);
-    if (i == 0) {
-        cp_async16(slots + (2 * NMAX) * kPipeThreads, reinterpret_cast<const float4*>(a.h) + q);
-        cp_async16(slots + (2 * NMAX + 1) * kPipeThreads, reinterpret_cast<const float4*>(a.c) + q);
-    }
-}
-
-template <int NMAX, bool LOSS>
-__global__ void __launch_bounds__(kPipeThreads, (NMAX >= 16 ? 3 : 6)) sync_step_pipe_kernel(const SyncStepParams p)
-{
-    extern __shared__ float4 pipe_smem[];
-    float4* slots = pipe_smem + threadIdx.x;  // slot s of this thread: slots[s * kPipeThreads]
-    const AvgParams& a = p.avg;
-    const float nf = (float)a.n;
-    const bool wd = p.wd != 0.0f;
-    double accD = 0.0, accL = 0.0;
-    bool redo = false;
-    const int64_t stride = (int64_t)gridDim.x * kPipeThreads;
-    const int64_t q_first = (int64_t)blockIdx.x * kPipeThreads + threadIdx.x;
-#pragma unroll
-    for (int i = 0; i < NMAX; ++i) {
-        pipe_fill<NMAX>(p, slots, q_first, i);
-        cp_async_commit();
-    }
-    for (int64_t q = q_first; q < a.Q; q += stride) {
-        const int64_t q_next = q + stride;
-        float4 xv[NMAX];
-        float4 hv = make_float4(0.0f, 0.0f, 0.0f, 0.0f), cv = hv;
-#pragma unroll
-        for (int i = 0; i < NMAX; ++i) {
-            // Commit groups in flight: (q, i .. NMAX-1) then (q_next, 0 .. i-1); the oldest is (q, i).
-            cp_async_wait<NMAX - 1>();
-            if (i < a.n) {
-                if (i == 0) {
-                    hv = slots[(2 * NMAX) * kPipeThreads];
-                    cv = slots[(2 * NMAX + 1) * kPipeThreads];
-                }
-                float4 x = slots[(2 * i) * kPipeThreads];
-                float4 v = slots[(2 * i + 1) * kPipeThreads];
-                const float4 z = normals4(p.keys, (uint32_t)q + p.q0, (uint32_t)i, p.k, 0u);
-                if (wd) {
-                    sgd_update<true>(x.x, v.x, hv.x, cv.x, z.x, p.gamma, p.mu, p.wd, p.sigma);
-                    sgd_update<true>(x.y, v.y, hv.y, cv.y, z.y, p.gamma, p.mu, p.wd, p.sigma);
-                    sgd_update<true>(x.z, v.z, hv.z, cv.z, z.z, p.gamma, p.mu, p.wd, p.sigma);
-                    sgd_update<true>(x.w, v.w, hv.w, cv.w, z.w, p.gamma, p.mu, p.wd, p.sigma);
-                } else {
-                    sgd_update<false>(x.x, v.x, hv.x, cv.x, z.x, p.gamma, p.mu, p.wd, p.sigma);
-                    sgd_update<false>(x.y, v.y, hv.y, cv.y, z.y, p.gamma, p.mu, p.wd, p.sigma);
-                    sgd_update<false>(x.z, v.z, hv.z, cv.z, z.z, p.gamma, p.mu, p.wd, p.sigma);
-                    sgd_update<false>(x.w, v.w, hv.w, cv.w, z.w, p.gamma, p.mu, p.wd, p.sigma);
-                }
-                reinterpret_cast<float4*>(p.v + (int64_t)i * a.P)[q] = v;
-                xv[i] = x;
-            } else {
-                xv[i] = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
-            }
-            // The slots of replica i have been read (the update used them): refill them.
-            pipe_fill<NMAX>(p, slots, q_next, i);
-            cp_async_commit();
-        }
-        redo |= !finish_group<NMAX, true, LOSS, true, true>(a, q, xv, nf, accD, accL);
-    }
-    cp_async_wait<0>();
-    if (redo)
-        for (int64_t q = q_first; q < a.Q; q += stride) redo_group<true, LOSS, true>(a, q, nf, accD, accL);
-    finish_sums_n<LOSS, kPipeThreads>(a, accD, accL);
-}
-
 using SyncStepKernel = void (*)(const SyncStepParams);
 
 template <int NMAX>
@@ -205,42 +108,12 @@ SyncStepKernel pick_nmax(bool bf16, bool loss)
     return loss ? sync_step_kernel<NMAX, false, true> : sync_step_kernel<NMAX, false, false>;
 }
 
-// The launch form of a shape: the kernel, its block size and its dynamic shared memory.
-struct SyncStepForm {
-    SyncStepKernel kernel;
-    int threads;
-    size_t smem;
-};
-
-template <int NMAX>
-SyncStepForm pipe_form(bool loss)
+SyncStepKernel pick(int32_t n, bool bf16, bool loss)
 {
-    const size_t smem = (size_t)pipe_slots<NMAX>() * kPipeThreads * sizeof(float4);
-    return {loss ? sync_step_pipe_kernel<NMAX, true> : sync_step_pipe_kernel<NMAX, false>, kPipeThreads, smem};
-}
-
-// Philox noise with 3 to 16 replicas: the pipelined form.  Otherwise (up to 2 replicas, or the
-// bf16 noise tensor) the register-resident form.
-SyncStepForm pick(int32_t n, bool bf16, bool loss)
-{
-    if (!bf16 && n >= 3) {
-        if (n <= 4) return pipe_form<4>(loss);
-        if (n <= 8) return pipe_form<8>(loss);
-        return pipe_form<16>(loss);
-    }
-    SyncStepKernel k;
-    if (n <= 2) k = pick_nmax<2>(bf16, loss);
-    else if (n <= 4) k = pick_nmax<4>(bf16, loss);
-    else if (n <= 8) k = pick_nmax<8>(bf16, loss);
-    else k = pick_nmax<16>(bf16, loss);
-    return {k, kThreads, 0};
-}
-
-// Dynamic shared memory above the default 48 KB must be allowed per kernel before its launch.
-cudaError_t allow_smem(const SyncStepForm& f)
-{
-    if (f.smem <= 48 * 1024) return cudaSuccess;
-    return cudaFuncSetAttribute(f.kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)f.smem);
+    if (n <= 2) return pick_nmax<2>(bf16, loss);
+    if (n <= 4) return pick_nmax<4>(bf16, loss);
+    if (n <= 8) return pick_nmax<8>(bf16, loss);
+    return pick_nmax<16>(bf16, loss);
 }
 
 }  // namespace
@@ -259,15 +132,13 @@ bool sync_step_supported(int32_t n, int64_t P, const void* x, const void* v, con
 
 int sync_step_grid(int32_t n, int64_t P, bool bf16, bool loss, int sms)
 {
-    const SyncStepForm f = pick(n, bf16, loss);
     int per_sm = 0;
-    if (allow_smem(f) != cudaSuccess ||
-        cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, f.kernel, f.threads, f.smem) != cudaSuccess ||
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, pick(n, bf16, loss), kThreads, 0) != cudaSuccess ||
         per_sm < 1) {
         cudaGetLastError();
         per_sm = 1;
     }
-    const int64_t work = (P / 4 + f.threads - 1) / f.threads;
+    const int64_t work = (P / 4 + kThreads - 1) / kThreads;
     int64_t grid = (int64_t)per_sm * sms;
     if (grid > work) grid = work;
     if (grid < 1) grid = 1;
@@ -296,10 +167,8 @@ cudaError_t launch_sync_step(const SyncStepArgs& s, cudaStream_t stream)
     p.wd = s.wd;
     p.sigma = s.sigma;
     p.keys = *s.keys;
-    const SyncStepForm f = pick(s.n, s.noise_bf16 != nullptr, s.loss);
-    const cudaError_t e = allow_smem(f);
-    if (e != cudaSuccess) return e;
-    f.kernel<<<(unsigned)s.grid, f.threads, f.smem, stream>>>(p);
+    const SyncStepKernel kernel = pick(s.n, s.noise_bf16 != nullptr, s.loss);
+    kernel<<<(unsigned)s.grid, kThreads, 0, stream>>>(p);
     return cudaGetLastError();
 }
 

@@ -82,11 +82,9 @@ def test_noise_modes_weight_decay_and_no_loss(bf16, wd, loss):
 
 
 @pytest.mark.parametrize("n", [3, 4, 6, 8])
-def test_pipelined_form_with_several_groups_per_thread(n):
-    # With Philox noise and 3..8 replicas the fused step runs the pipelined form (asynchronous
-    # copies into shared memory, refilled for the next group while a group is stepped and
-    # averaged).  At 2^20 + 148 columns every thread of its persistent grid takes two or three
-    # groups, so the refills are consumed: whole runs bit-exact against the oracle.
+def test_several_groups_per_thread(n):
+    # At 2^20 + 148 columns every thread of the fused step's persistent grid takes several column
+    # groups in its grid-stride loop: whole runs bit-exact against the oracle (all host cores).
     P, K = (1 << 20) + 4 * 37, 12
     w = inputs.WORKLOADS["resnet18-n8"]
     h, c = inputs.draw_h(P, w.h_dist, 8), inputs.draw_c(P, 1.0, 8)
