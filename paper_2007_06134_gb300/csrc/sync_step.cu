@@ -47,7 +47,9 @@ struct SyncStepParams {
 // - a tile per block with a barrier, each thread stepping two (replica, group) items and then
 //   averaging whole columns of the tile: 0.469 ms (400 M instructions);
 // - per-warp bulk copies (cp.async.bulk on mbarriers, lane 0 refilling a 3-stage ring): 0.396 ms
-//   (351 M instructions, most of the excess in the waits).
+//   (351 M instructions, most of the excess in the waits);
+// - v loaded one replica ahead instead of with x (78 registers, 3 blocks of 256 per SM): 0.75 of
+//   the copy peak at n = 8, P = 2^26, against 0.79 here.
 template <int NMAX, bool BF16, bool LOSS>
 __global__ void __launch_bounds__(kThreads, (NMAX >= 16 ? 1 : 2)) sync_step_kernel(const SyncStepParams p)
 {
