@@ -219,6 +219,12 @@ void orc_box_muller_words(uint32_t w_radius, uint32_t w_angle, float* z0, float*
     box_muller(w_radius, w_angle, z0, z1);
 }
 
+/* The same over arrays of word pairs (for exhaustive comparisons). */
+void orc_box_muller_array(const uint32_t* w_radius, const uint32_t* w_angle, int64_t m, float* z0, float* z1)
+{
+    for (int64_t t = 0; t < m; ++t) box_muller(w_radius[t], w_angle[t], &z0[t], &z1[t]);
+}
+
 /* The four normals of one Philox block: words (0,1) -> elements 4q+0, 4q+1, */
 /* words (2,3) -> elements 4q+2, 4q+3.                                       */
 static void normals_of_block(uint64_t seed, uint32_t tag, uint32_t i, uint32_t k, uint64_t q, float z[4])

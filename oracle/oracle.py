@@ -111,6 +111,8 @@ def lib():
                                       C.c_int64, C.POINTER(C.c_float)]
             L.orc_box_muller_words.argtypes = [C.c_uint32, C.c_uint32, C.POINTER(C.c_float),
                                                C.POINTER(C.c_float)]
+            L.orc_box_muller_array.argtypes = [C.POINTER(C.c_uint32), C.POINTER(C.c_uint32), C.c_int64,
+                                               C.POINTER(C.c_float), C.POINTER(C.c_float)]
             L.orc_to_bf16_array.argtypes = [C.POINTER(C.c_float), C.POINTER(C.c_uint16), C.c_int64]
             L.orc_noise_bf16.argtypes = [C.c_uint64, C.c_int32, C.c_int64, C.POINTER(C.c_uint16)]
             L.orc_local_step.argtypes = [C.c_int32, C.c_int64, C.c_int64, C.c_int64,
@@ -197,6 +199,16 @@ def box_muller_words(w_radius: int, w_angle: int):
     z1 = C.c_float()
     lib().orc_box_muller_words(w_radius, w_angle, C.byref(z0), C.byref(z1))
     return z0.value, z1.value
+
+
+def box_muller_array(w_radius, w_angle):
+    """(z0, z1) arrays of Box-Muller on word pairs: radius sqrt(-2 ln u1), angle 2 pi u2."""
+    wr = np.ascontiguousarray(w_radius, dtype=np.uint32)
+    wa = np.ascontiguousarray(w_angle, dtype=np.uint32)
+    z0 = np.empty(wr.size, np.float32)
+    z1 = np.empty(wr.size, np.float32)
+    lib().orc_box_muller_array(_u32p(wr), _u32p(wa), wr.size, _f32p(z0), _f32p(z1))
+    return z0, z1
 
 
 def to_bf16(x) -> np.ndarray:

@@ -145,7 +145,8 @@ __global__ void __launch_bounds__(kStepThreads) local_step_kernel(const StepPara
 // by the last block to finish, in block order, so the sums do not depend on which block
 // finishes last.
 template <int NMAX, int U, bool VEC, bool LOSS, bool WRITE>
-__global__ void __launch_bounds__(kThreads, (NMAX <= 8 ? 4 : (NMAX >= 32 ? 1 : 2))) average_kernel(const AvgParams p)
+__global__ void __launch_bounds__(kThreads, ((NMAX == 2 || (NMAX <= 8 && U == 1)) ? 4 : (NMAX >= 32 ? 1 : 2)))
+    average_kernel(const AvgParams p)
 {
     using G = ColumnGroup<VEC>;
     using T = typename G::T;
@@ -259,19 +260,22 @@ AvgKernel pick_average_nmax(bool vec, bool loss, bool write)
 }
 
 // Register-resident variants: NMAX replicas x U column groups per thread (NMAX * U <= 32 float4).
-// Resident blocks per SM (the register cap): 4 for n <= 8, 1 for n <= 32 and 2 otherwise.  With
+// Resident blocks per SM (the register cap): 4 for n <= 2 and for one group per thread up to 8
+// replicas, 1 for n <= 32 and 2 otherwise.  With
 // two rows per column a thread has few bytes in flight, so n <= 2 takes 4 blocks of 4 groups:
 // measured 0.93 of the copy peak at P = 2^28, against 0.71 with 2 blocks.  Its loss variant takes
 // 2 groups, which fit the 64 registers of that cap without spilling.  For 3 to 8 replicas, 4
 // blocks of one group per thread measured (L2 flushed; P = 2^22 / 2^24 / 2^26 / 2^28)
 // 0.79 / 0.92 / 0.96 / 0.96 of the copy peak at n = 4 and 0.89 / 0.92 / 0.93 / 0.94 at n = 8, against
-// 0.65 / 0.87 / 0.95 / 0.98 and 0.85 / 0.91 / 0.92 / 0.92 with 2 blocks of 4 and of 2 groups.  For 16
-// replicas 3 blocks measured 0.89-0.90 against 0.92 with 2.
+// 0.65 / 0.87 / 0.95 / 0.98 and 0.85 / 0.91 / 0.92 / 0.92 with 2 blocks of 4 and of 2 groups.  With
+// the loss (h and c read too) the one-group form measured slower right after a local step (0.92
+// against 0.96 of the peak on 8 replicas of 138 M columns), so the loss variants keep 2 blocks of
+// 4 (n <= 4) and 2 (n <= 8) groups.  For 16 replicas 3 blocks measured 0.89-0.90 against 0.92 with 2.
 AvgKernel pick_average(int32_t n, bool vec, bool loss, bool write)
 {
     if (n <= 2) return pick_average_nmax<2, 4, 2>(vec, loss, write);
-    if (n <= 4) return pick_average_nmax<4, 1>(vec, loss, write);
-    if (n <= 8) return pick_average_nmax<8, 1>(vec, loss, write);
+    if (n <= 4) return pick_average_nmax<4, 1, 4>(vec, loss, write);
+    if (n <= 8) return pick_average_nmax<8, 1, 2>(vec, loss, write);
     if (n <= 16) return pick_average_nmax<16, 1>(vec, loss, write);
     if (n <= 32) return pick_average_nmax<32, 1>(vec, loss, write);
     return pick_average_nmax<0, 1>(vec, loss, write);
