@@ -122,7 +122,7 @@ SyncStepKernel pick(int32_t n, bool bf16, bool loss)
 
 // Used where it measured faster than the two kernels it replaces: up to 8 replicas, and up to 16
 // with the pre-materialised bf16 noise.  With Philox noise and 9..16 replicas the 16-replica form
-// (one block per SM, 8 warps) measured 0.04 to 0.41 ms slower per sync from P = 2^22 to 2^26.
+// (one block per SM, 8 warps) measured 0.01 to 0.23 ms slower per sync from P = 2^22 to 2^26.
 bool sync_step_supported(int32_t n, int64_t P, const void* x, const void* v, const void* h, const void* c,
                          const void* noise_bf16)
 {
