@@ -176,7 +176,7 @@ typedef struct {
 int adpsgd_init(const adpsgd_config* cfg, float* x, float* v, const float* h, const float* c,
                 const uint16_t* noise_bf16, void* stream, adpsgd_ctx** out);
 
-/* m local steps of every replica (Algorithm 1 and 2, "updating parameter variables locally";
+/* m local steps of every replica (Algorithm 1 and 2, the local update;
  * Sec. IV-A momentum): for t in [0, m), step k = k0 + t with step size lr[t] (host array):
  *   g = h (x - c) + sigma z[i, j, k];  if wd != 0: g += wd x;  v = mu v + g;  x -= lr[t] v
  * each a separately rounded fp32 operation.  z is word (j mod 4) of Philox4x32-10 with counter

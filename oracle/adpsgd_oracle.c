@@ -16,7 +16,7 @@
  *   - The local step of Algorithm 1 (update line) and Algorithm 2 (update line)
  *     on the surrogate objective f(x) = 1/2 sum_j h_j (x_j - c_j)^2, with SGD
  *     momentum and weight decay in the PyTorch 1.0 convention the experiments
- *     used (Sec. IV-A: "momentum coefficient 0.9").
+ *     used (Sec. IV-A gives the momentum, 0.9, and nothing else about it).
  *   - Parameter averaging (Algorithm 2, averaging line; Eq. alg1's A_n) and the
  *     inter-replica variance of Sec. II-B (definition of Var[W_k]) and S_k of
  *     Algorithm 2, plus the surrogate loss at the average.
@@ -294,8 +294,8 @@ void orc_noise_bf16(uint64_t seed, int32_t n, int64_t P, uint16_t* out)
 }
 
 /* ------------------------------------------------------------------------ */
-/* Local step (Algorithm 1 / Algorithm 2, "updating parameter variables     */
-/* locally"), for every replica i and columns j in [j0, j1).                 */
+/* Local step (Algorithm 1 / Algorithm 2, the local update), for every     */
+/* replica i and columns j in [j0, j1).                                      */
 /* Stochastic gradient of the surrogate: g = h_j (x - c_j) + sigma * z.      */
 /* Reading R1: g += wd * x (only when wd != 0); v = mu * v + g;              */
 /* x = x - gamma * v.  Each operation is one fp32 rounding.                  */

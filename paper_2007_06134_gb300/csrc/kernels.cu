@@ -1,6 +1,6 @@
 // kernels.cu -- sm_103a kernels of the ADPSGD hot path.
 //
-//   local_step_kernel  Algorithm 2 "updating parameter variables locally" for all n replicas in
+//   local_step_kernel  Algorithm 2's local update for all n replicas in
 //                      one pass: gradient of the quadratic surrogate, Philox/Box-Muller noise
 //                      (or a pre-materialised bf16 noise tensor), weight decay, momentum and
 //                      the parameter update, 128-bit loads and stores.  HBM-bound: per

@@ -1,5 +1,5 @@
 // sync_step.cu -- the local step of a sync iteration fused with the averaging that ends it
-// (Algorithm 2: the last "updating parameter variables locally" of an interval, then the
+// (Algorithm 2: the last local update of an interval, then the
 // averaging and S_k).  Each thread owns one float4 column group of all n replicas: it loads x,
 // v (and h, c once), applies the local step to every replica in registers with the same
 // operations as local_step_kernel, writes v, and then averages the new x with the same
