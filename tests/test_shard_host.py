@@ -168,3 +168,49 @@ def test_replica_split_collectives_between_two_gloo_processes():
         scattered, x_after = got[r]
         assert np.array_equal(scattered, x_all[:, c0:c0 + cols])
         assert np.array_equal(x_after, np.repeat(mean_row[None, :], x_after.shape[0], axis=0))
+
+
+def _leaving_worker(rank, world, port, q):
+    os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port), RANK=str(rank), WORLD_SIZE=str(world))
+    sys.path.insert(0, ROOT)
+    import datetime
+
+    import torch.distributed as dist
+
+    from paper_2007_06134_gb300 import abi as A
+    from paper_2007_06134_gb300 import shard as S
+    dist.init_process_group("gloo", rank=rank, world_size=world, timeout=datetime.timedelta(seconds=20))
+    group = dist.new_group(backend="gloo", timeout=datetime.timedelta(seconds=5))
+    cb, _ = S.dist_gather(group)
+    def report(value):
+        q.put((rank, value))
+        q.close()
+        q.join_thread()  # the message is sent before the process ends
+
+    if rank == 1:
+        report("left")
+        os._exit(0)  # this rank leaves between syncs, without a word to the others
+    sh = A.make_shard(world, rank, 0, 8, cb)
+    try:
+        A.adpsgd_shard_combine(sh, [1.0, 2.0])
+        report("no error")
+    except A.AdpsgdError as e:
+        report(e.status)
+    os._exit(0)
+
+
+def test_a_rank_that_leaves_is_reported_as_a_peer_failure():
+    # Failure detection on the host: when a shard's process is gone, the exchange runs out its
+    # process-group timeout and the library reports ADPSGD_E_PEER instead of hanging.
+    import torch.multiprocessing as mp
+    ctx = mp.get_context("spawn")
+    q = ctx.Queue()
+    port = _free_port()
+    procs = [ctx.Process(target=_leaving_worker, args=(r, 2, port, q)) for r in range(2)]
+    for p in procs:
+        p.start()
+    got = dict(q.get(timeout=120) for _ in range(2))
+    for p in procs:
+        p.join(60)
+    assert got[1] == "left"
+    assert got[0] == abi.E_PEER
