@@ -49,7 +49,11 @@ struct SyncStepParams {
 // - per-warp bulk copies (cp.async.bulk on mbarriers, lane 0 refilling a 3-stage ring): 0.396 ms
 //   (351 M instructions, most of the excess in the waits);
 // - v loaded one replica ahead instead of with x (78 registers, 3 blocks of 256 per SM): 0.75 of
-//   the copy peak at n = 8, P = 2^26, against 0.79 here.
+//   the copy peak at n = 8, P = 2^26, against 0.79 here;
+// - (after the generator's fma division and square root, which brought this form to 0.85 there)
+//   the replicas in a loop that is not unrolled, the next replica's x and v loaded into registers
+//   while one is stepped, the new x in per-thread shared-memory slots: 0.77-0.79 at 6 or 8 blocks
+//   of 128 per SM.
 template <int NMAX, bool BF16, bool LOSS>
 __global__ void __launch_bounds__(kThreads, (NMAX >= 16 ? 1 : 2)) sync_step_kernel(const SyncStepParams p)
 {
