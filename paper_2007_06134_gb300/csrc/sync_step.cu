@@ -30,8 +30,9 @@ struct SyncStepParams {
 };
 
 // Register cap: 128 per thread (2 blocks of 256 per SM) up to 8 replicas, 255 for 16.  One
-// thread per column group.  Other forms measured slower on resnet18-n8 (0.314 ms here, one launch
-// under ncu; 225 M warp-instructions at 60 % issue):
+// thread per column group.  Other forms measured slower on resnet18-n8 than this one did at the
+// time (0.314 ms, one launch under ncu, 225 M warp-instructions at 60 % issue; 0.294 ms and 213 M
+// since the generator's fma division and square root):
 // - splitting a group's replicas over two lanes that swap halves by shuffles (0.346 ms);
 // - a tiled form, with a thread per (group, replica) as in local_step_kernel and the averaging
 //   from a shared-memory tile (0.350 ms);
