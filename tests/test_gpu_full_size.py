@@ -1,8 +1,9 @@
 """Parity at the workloads' full sizes, in the launch configuration the bench times.
 
-The adaptive runs the bench times (Algorithm 2, p_init 4, K_s = K / 4, fused sync steps, the loss
-at every sync) are compared with the oracle's chunked all-core run over all columns at every
-sync: k, p and the phase bit-exact, S, the loss and C_2 within 1e-4, the final x and v bit-exact.
+The adaptive runs the bench times (Algorithm 2, p_init 4, K_s = K / 4, the loss at every sync;
+with fused sync steps, and with fused intervals) are compared with the oracle's chunked all-core
+run over all columns at every sync: k, p and the phase bit-exact, S, the loss and C_2 within
+1e-4, the final x and v bit-exact.
 
 The surrogate objective is separable per column and the constant-period schedule does not
 depend on the data, so the oracle can also follow a full-size constant-period run exactly on a
@@ -174,32 +175,41 @@ FULL_RUN_K = {"resnet18-n8": 2000, "vgg16-n8": 100, "resnet50-n16-bf16noise": 20
 
 @pytest.mark.parametrize("name", list(FULL_RUN_K))
 def test_full_size_adaptive_run_against_oracle_at_every_sync(name):
+    # Both launch forms the bench times: fused sync steps (the headline) and fused intervals (its
+    # fused_intervals figure), each against one oracle run.
     w = inputs.WORKLOADS[name]
     K = FULL_RUN_K[name]
     if K != w.K:
         w = dataclasses.replace(w, K=K, milestones=tuple(m * K // w.K for m in w.milestones))
     bf16 = w.noise == "bf16"
     h, c = inputs.problem(w)
-    # GPU: the bench's launch configuration
-    xd = torch.zeros((w.n, w.P), dtype=torch.float32, device=DEV)
-    vd = torch.zeros_like(xd)
+    sched = abi.make_schedule(abi.ADPSGD, w.K, w.p_init, K_s=w.K_s, lr0=w.lr0, lr_factor=w.lr_factor,
+                              milestones=w.milestones)
+    runs = {}
+    hd, cd = _dev(h), _dev(c)
     nd = None
     if bf16:
         nd = torch.empty((w.n, w.P), dtype=torch.int16, device=DEV)
         abi.adpsgd_noise_fill_bf16(w.seed, w.n, w.P, nd)
-    sched = abi.make_schedule(abi.ADPSGD, w.K, w.p_init, K_s=w.K_s, lr0=w.lr0, lr_factor=w.lr_factor,
-                              milestones=w.milestones)
-    tr = abi.TraceBuffers(w.K)
-    cfg = abi.make_config(w.n, w.P, momentum=w.mu, weight_decay=w.wd, noise_sigma=w.sigma, seed=w.seed,
-                          noise_mode=abi.NOISE_BF16 if bf16 else abi.NOISE_PHILOX, want_loss=True,
-                          fuse_sync_step=True)
-    with abi.adpsgd_init(cfg, xd, vd, _dev(h), _dev(c), nd) as ctx:
-        stats = abi.adpsgd_run(ctx, sched, abi.adpsgd_state_init(sched), trace=tr)
-    torch.cuda.synchronize()
-    assert stats.sync_step_launches > 0 and stats.sync_step_launches + stats.average_launches == stats.rounds
-    gx, gv = xd.cpu().numpy(), vd.cpu().numpy()
-    del xd, vd, nd
-    torch.cuda.empty_cache()
+    for mode in ("sync_step", "intervals"):
+        xd = torch.zeros((w.n, w.P), dtype=torch.float32, device=DEV)
+        vd = torch.zeros_like(xd)
+        tr = abi.TraceBuffers(w.K)
+        cfg = abi.make_config(w.n, w.P, momentum=w.mu, weight_decay=w.wd, noise_sigma=w.sigma, seed=w.seed,
+                              noise_mode=abi.NOISE_BF16 if bf16 else abi.NOISE_PHILOX, want_loss=True,
+                              fuse_sync_step=mode == "sync_step", fuse_intervals=mode == "intervals")
+        with abi.adpsgd_init(cfg, xd, vd, hd, cd, nd) as ctx:
+            stats = abi.adpsgd_run(ctx, sched, abi.adpsgd_state_init(sched), trace=tr)
+        torch.cuda.synchronize()
+        if mode == "sync_step":
+            assert stats.sync_step_launches > 0
+            assert stats.sync_step_launches + stats.average_launches == stats.rounds
+        else:
+            assert stats.interval_launches >= stats.rounds > 0
+        runs[mode] = (stats, tr.arrays(), xd.cpu().numpy(), vd.cpu().numpy())
+        del xd, vd
+        torch.cuda.empty_cache()
+    del hd, cd, nd
     # oracle: the same run over all columns on every host core
     x, v = inputs.zero_state(w.n, w.P)
     noise = O.noise_bf16(w.seed, w.n, w.P) if bf16 else None
@@ -207,7 +217,6 @@ def test_full_size_adaptive_run_against_oracle_at_every_sync(name):
                           milestones=w.milestones)
     otr = O.run(x, v, h, c, spec=spec, seed=w.seed, mu=w.mu, wd=w.wd, sigma=w.sigma, noise=noise,
                 threads=O.host_threads())
-    t = tr.arrays()
     # every adaptive decision well away from the thresholds, so that the bit-exact comparison of
     # the schedule is well posed (S agrees to far better than 1e-6)
     C2_before = np.concatenate([[0.0], otr.C2[:-1]])
@@ -215,14 +224,15 @@ def test_full_size_adaptive_run_against_oracle_at_every_sync(name):
         if ph == O.PHASE_ADAPTING and C2b > 0.0:
             ratio = S / (np.float64(O.gamma(spec, int(k))) * C2b)
             assert min(abs(ratio - 0.7) / 0.7, abs(ratio - 1.3) / 1.3) > 1e-6, (name, k, ratio)
-    assert stats.rounds == otr.syncs == len(t["k"])
-    assert np.array_equal(t["k"], otr.k) and np.array_equal(t["p"], otr.p)
-    assert np.array_equal(t["phase"], otr.phase)
-    for key in ("S", "loss", "C2"):
-        for s_idx, (a, b) in enumerate(zip(t[key], getattr(otr, key))):
-            assert _rel(a, b) < REL or (a == 0.0 and b == 0.0), (name, key, s_idx, a, b)
-    assert np.array_equal(gx.view(np.uint32), x.view(np.uint32)), name
-    assert np.array_equal(gv.view(np.uint32), v.view(np.uint32)), name
+    for mode, (stats, t, gx, gv) in runs.items():
+        assert stats.rounds == otr.syncs == len(t["k"]), mode
+        assert np.array_equal(t["k"], otr.k) and np.array_equal(t["p"], otr.p), mode
+        assert np.array_equal(t["phase"], otr.phase), mode
+        for key in ("S", "loss", "C2"):
+            for s_idx, (a, b) in enumerate(zip(t[key], getattr(otr, key))):
+                assert _rel(a, b) < REL or (a == 0.0 and b == 0.0), (name, mode, key, s_idx, a, b)
+        assert np.array_equal(gx.view(np.uint32), x.view(np.uint32)), (name, mode)
+        assert np.array_equal(gv.view(np.uint32), v.view(np.uint32)), (name, mode)
 
 
 def _cfg_big(n, P, mu, wd, sigma, seed, mode):
