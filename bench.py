@@ -607,6 +607,45 @@ def run_sweep(args):
             del xd
 
 
+def run_local_sweep(args):
+    """The local step alone over n x P (Philox noise, weight decay): each point times 20 launches
+    with CUDA events, every launch after a write-then-read L2 flush; GB/s on 16 n P + 8 P bytes."""
+    import torch
+
+    from paper_2007_06134_gb300 import abi, inputs
+    peak, peak_kind = measured_peaks()
+    device = torch.device("cuda", 0)
+    stream = torch.cuda.current_stream(device)
+    l2 = torch.cuda.get_device_properties(device).L2_cache_size
+    flush = torch.empty(int(2 * l2) // 4, dtype=torch.float32, device=device)
+    w = inputs.WORKLOADS["resnet18-n8"]
+    for n in (2, 4, 8, 16, 32):
+        for lp in (20, 22, 24, 26, 28):
+            P = 1 << lp
+            if (16 * n + 8) * P > args.sweep_max_bytes:
+                continue
+            h, c = inputs.problem(w, P)
+            hd, cd = torch.from_numpy(h).to(device), torch.from_numpy(c).to(device)
+            xd = torch.zeros((n, P), dtype=torch.float32, device=device)
+            vd = torch.zeros_like(xd)
+            cfg = abi.make_config(n, P, momentum=w.mu, weight_decay=w.wd, noise_sigma=w.sigma, seed=w.seed,
+                                  time_kernels=1)
+            with abi.adpsgd_init(cfg, xd, vd, hd, cd, None, stream) as ctx:
+                abi.adpsgd_local_steps(ctx, 0, [w.lr0] * 3)
+                abi.adpsgd_reset_kernel_times(ctx)
+                for k in range(20):
+                    flush.zero_()
+                    flush.sum()
+                    abi.adpsgd_local_steps(ctx, 3 + k, [w.lr0])
+                t = abi.adpsgd_kernel_times(ctx)
+            ms = t["local_step_ms"] / t["local_step_launches"]
+            gbs = (16 * n + 8) * P / (ms / 1e3) / 1e9
+            print(json.dumps({"sweep": "local_step", "n": n, "P": P, "ms": ms, "GB/s": gbs, "frac": gbs / peak,
+                              "peak": peak, "peak_kind": peak_kind, "l2_flushed": "write then read a 2 x L2 buffer",
+                              "replica_params_per_s": n * P / (ms / 1e3)}), flush=True)
+            del xd, vd, hd, cd
+
+
 def run_sync_sweep(args):
     """The fused sync step against the local step and the averaging it replaces, over n x P: a
     CPSGD p = 2 run (every other iteration ends with a sync) with every launch timed, once with
@@ -739,6 +778,7 @@ def main():
     ap.add_argument("--sweep", action="store_true", help="averaging-kernel sweep over n x P instead")
     ap.add_argument("--sync-sweep", action="store_true",
                     help="fused sync step against the local step + averaging over n x P instead")
+    ap.add_argument("--local-sweep", action="store_true", help="the local step alone over n x P instead")
     ap.add_argument("--sweep-max-bytes", type=float, default=70e9)
     ap.add_argument("--variance-traces", action="store_true",
                     help="the schedule study of Sec. III with per-iteration variance instead")
@@ -755,6 +795,8 @@ def main():
         return run_sweep(args)
     if args.sync_sweep:
         return run_sync_sweep(args)
+    if args.local_sweep:
+        return run_local_sweep(args)
     if args.variance_traces:
         return run_variance_traces(args)
     return run_gpu(args, w)
