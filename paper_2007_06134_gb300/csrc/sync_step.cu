@@ -54,7 +54,12 @@ struct SyncStepParams {
 // - (after the generator's fma division and square root, which brought this form to 0.85 there)
 //   the replicas in a loop that is not unrolled, the next replica's x and v loaded into registers
 //   while one is stepped, the new x in per-thread shared-memory slots: 0.77-0.79 at 6 or 8 blocks
-//   of 128 per SM.
+//   of 128 per SM;
+// - teams of 8 lanes over two column groups, lane i stepping replica i as local_step_kernel does
+//   (80 registers, 3 blocks of 256 per SM), the new x through a shared-memory tile and lane j
+//   then taking column j's mean and squared deviations, with shuffles for the group sums: 0.360 ms
+//   under ncu, 306 M instructions (per-lane statistics, shuffles and h, c loads), 0.56 of the copy
+//   peak at n = 8, P = 2^26, and 0.45 with bf16 noise; 4 blocks per SM (64 registers) was slower.
 template <int NMAX, bool BF16, bool LOSS>
 __global__ void __launch_bounds__(kThreads, (NMAX >= 16 ? 1 : 2)) sync_step_kernel(const SyncStepParams p)
 {
