@@ -564,7 +564,9 @@ def run_gpu(args, w):
 
 
 def run_sweep(args):
-    """Averaging + variance alone over n x P (the sweep workload): GB/s and fraction of peak per point."""
+    """Averaging + variance alone over n x P (the sweep workload): GB/s and fraction of peak per point.
+    Every launch starts from distinct replicas (restored from a copy, then the L2 flushed): the
+    averaging leaves identical replicas behind, which is not the state a sync finds."""
     import torch
 
     from paper_2007_06134_gb300 import abi, inputs
@@ -586,16 +588,19 @@ def run_sweep(args):
             P = 1 << lp
             if 8 * n * P > args.sweep_max_bytes:
                 continue
-            xd = torch.randn((n, P), dtype=torch.float32, device=device)
-            xd += torch.arange(n, device=device, dtype=torch.float32)[:, None] * 1e-3
+            x0 = torch.randn((n, P), dtype=torch.float32, device=device)
+            x0 += torch.arange(n, device=device, dtype=torch.float32)[:, None] * 1e-3
+            xd = torch.empty_like(x0)
             z = torch.zeros(P, device=device)
             cfg = abi.make_config(n, P, want_loss=False, time_kernels=True)
             with abi.adpsgd_init(cfg, xd, xd, z, z, None, stream) as ctx:
                 reps = max(5, min(50, int(2e10 // (8 * n * P))))
                 for _ in range(3):
+                    xd.copy_(x0)
                     abi.adpsgd_average_and_variance(ctx, want_loss=False)
                 abi.adpsgd_reset_kernel_times(ctx)
                 for _ in range(reps):
+                    xd.copy_(x0)
                     flush_l2()
                     abi.adpsgd_average_and_variance(ctx, want_loss=False)
                 t = abi.adpsgd_kernel_times(ctx)
@@ -603,8 +608,9 @@ def run_sweep(args):
             gbs = 8 * n * P / (ms / 1e3) / 1e9
             print(json.dumps({"sweep": "average_and_variance", "n": n, "P": P, "ms": ms, "GB/s": gbs,
                               "frac": gbs / peak, "peak": peak, "peak_kind": peak_kind,
-                              "l2_flushed": "write then read a 2 x L2 buffer"}), flush=True)
-            del xd
+                              "l2_flushed": "write then read a 2 x L2 buffer",
+                              "replicas": "distinct at every launch"}), flush=True)
+            del xd, x0
 
 
 def run_local_sweep(args):

@@ -35,7 +35,7 @@ __device__ __forceinline__ void column_stats_global(const float* x, int64_t P, i
         spread = spread + fabsf(diff);
     }
     z = spread;
-    xbar = base + __fdiv_rn(acc, nf);
+    xbar = base + mean_offset(acc, nf);
     float s = 0.0f;
     for (int i = 0; i < n; ++i) {
         const float dev = x[(int64_t)i * P + j] - xbar;

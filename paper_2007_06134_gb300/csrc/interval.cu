@@ -67,7 +67,7 @@ __device__ __forceinline__ void column_stats_tile(const float4 (*tile)[kTileGrou
     const float base = reinterpret_cast<const float*>(&tile[0][g])[r];
     float acc = 0.0f;
     for (int j = 1; j < n; ++j) acc = acc + (reinterpret_cast<const float*>(&tile[j][g])[r] - base);
-    xbar = base + __fdiv_rn(acc, nf);
+    xbar = base + mean_offset(acc, nf);
     float s = 0.0f;
     for (int j = 0; j < n; ++j) {
         const float dev = reinterpret_cast<const float*>(&tile[j][g])[r] - xbar;
