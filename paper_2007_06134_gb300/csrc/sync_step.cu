@@ -30,9 +30,15 @@ struct SyncStepParams {
 };
 
 // Register cap: 128 per thread (2 blocks of 256 per SM) up to 8 replicas, 255 for 16.  One
-// thread per column group.  Other forms measured slower on resnet18-n8 than this one did at the
-// time (0.314 ms, one launch under ncu, 225 M warp-instructions at 60 % issue; 0.294 ms and 213 M
-// since the generator's fma division and square root):
+// thread per column group.  With Philox noise the n normals4 calls run first, in a loop that is
+// not unrolled, into per-thread shared-memory slots (NMAX x 256 float4 per block): the
+// generator's code is there once instead of n times, and its arithmetic runs while the loads of
+// x and v are in flight.  Against the same kernel with the generator unrolled into the update
+// (below the register-resident form of the list) it measured 0.93 against 0.84 of the copy peak
+// at n = 8, P = 2^26, 0.90 against 0.81 at 2^24 and 0.93 against 0.87 at n = 4, P = 2^26.
+// Other forms measured slower on resnet18-n8 than the unrolled form did at the time (0.314 ms,
+// one launch under ncu, 225 M warp-instructions at 60 % issue; 0.294 ms and 213 M since the
+// generator's fma division and square root):
 // - splitting a group's replicas over two lanes that swap halves by shuffles (0.346 ms);
 // - a tiled form, with a thread per (group, replica) as in local_step_kernel and the averaging
 //   from a shared-memory tile (0.350 ms);
@@ -63,6 +69,7 @@ struct SyncStepParams {
 template <int NMAX, bool BF16, bool LOSS>
 __global__ void __launch_bounds__(kThreads, (NMAX >= 16 ? 1 : 2)) sync_step_kernel(const SyncStepParams p)
 {
+    __shared__ float4 zs[BF16 ? 1 : NMAX][BF16 ? 1 : kThreads];  // thread t's normals of replica i: zs[i][t]
     const AvgParams& a = p.avg;
     const float nf = (float)a.n;
     const bool wd = p.wd != 0.0f;
@@ -82,6 +89,11 @@ __global__ void __launch_bounds__(kThreads, (NMAX >= 16 ? 1 : 2)) sync_step_kern
                 vv[i] = reinterpret_cast<const float4*>(p.v + row)[q];
                 if (BF16) nb[i] = __ldg(reinterpret_cast<const uint2*>(p.noise + row) + q);
             }
+        if (!BF16) {
+#pragma unroll 1
+            for (int i = 0; i < a.n; ++i)
+                zs[i][threadIdx.x] = normals4(p.keys, (uint32_t)q + p.q0, (uint32_t)i, p.k, 0u);
+        }
 #pragma unroll
         for (int i = 0; i < NMAX; ++i)
             if (i < a.n) {
@@ -89,7 +101,7 @@ __global__ void __launch_bounds__(kThreads, (NMAX >= 16 ? 1 : 2)) sync_step_kern
                                                     __uint_as_float(nb[i].x & 0xFFFF0000u),
                                                     bf16_bits_to_float(nb[i].y & 0xFFFFu),
                                                     __uint_as_float(nb[i].y & 0xFFFF0000u))
-                                      : normals4(p.keys, (uint32_t)q + p.q0, (uint32_t)i, p.k, 0u);
+                                      : zs[i][threadIdx.x];
                 if (wd) {
                     sgd_update<true>(xv[i].x, vv[i].x, hv.x, cv.x, z.x, p.gamma, p.mu, p.wd, p.sigma);
                     sgd_update<true>(xv[i].y, vv[i].y, hv.y, cv.y, z.y, p.gamma, p.mu, p.wd, p.sigma);
@@ -120,19 +132,22 @@ SyncStepKernel pick_nmax(bool bf16, bool loss)
     return loss ? sync_step_kernel<NMAX, false, true> : sync_step_kernel<NMAX, false, false>;
 }
 
+// 9..16 replicas: the bf16 noise tensor only (sync_step_supported).
 SyncStepKernel pick(int32_t n, bool bf16, bool loss)
 {
     if (n <= 2) return pick_nmax<2>(bf16, loss);
     if (n <= 4) return pick_nmax<4>(bf16, loss);
     if (n <= 8) return pick_nmax<8>(bf16, loss);
-    return pick_nmax<16>(bf16, loss);
+    return loss ? sync_step_kernel<16, true, true> : sync_step_kernel<16, true, false>;
 }
 
 }  // namespace
 
 // Used where it measured faster than the two kernels it replaces: up to 8 replicas, and up to 16
 // with the pre-materialised bf16 noise.  With Philox noise and 9..16 replicas the 16-replica form
-// (one block per SM, 8 warps) measured 0.01 to 0.23 ms slower per sync from P = 2^22 to 2^26.
+// (one block of 256 per SM, 234 registers, the generator loop included) measured 0.54-0.62 of
+// the copy peak at n = 9 and 12 against 0.56-0.64 for the two kernels from P = 2^22 to 2^26, and
+// 0.61-0.66 against 0.60-0.63 at n = 16.
 bool sync_step_supported(int32_t n, int64_t P, const void* x, const void* v, const void* h, const void* c,
                          const void* noise_bf16)
 {
