@@ -664,8 +664,9 @@ def run_sync_sweep(args):
     device = torch.device("cuda", 0)
     stream = torch.cuda.current_stream(device)
     w = inputs.WORKLOADS["resnet18-n8"]
-    # the shapes the fused step takes: up to 8 replicas with Philox noise, up to 16 with bf16 noise
-    for n, bf16 in ((2, False), (4, False), (6, False), (8, False), (8, True), (16, True)):
+    # the fused step's forms: registers up to 8 replicas, two halves for 9..16 with Philox noise,
+    # the 16-replica register form with the bf16 noise tensor
+    for n, bf16 in ((2, False), (4, False), (6, False), (8, False), (12, False), (16, False), (8, True), (16, True)):
         for lp in (22, 24, 26):
             P = 1 << lp
             h, c = inputs.problem(w, P)

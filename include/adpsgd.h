@@ -80,9 +80,9 @@ typedef struct {
                                 25 bytes per replica-param).  Bit-identical results (D and the
                                 loss up to the order of fp64 additions).  Valid for any objective
                                 whose gradient is computed per element in the step; nothing is
-                                carried across steps.  Used where it measured faster: n <= 8 (n <= 16
-                                with the bf16 noise tensor), P % 4 == 0, every array 16-byte aligned
-                                (bf16 noise: 8-byte); elsewhere ignored. */
+                                carried across steps.  Used where it measured faster: n <= 16,
+                                P % 4 == 0, every array 16-byte aligned (bf16 noise: 8-byte);
+                                elsewhere ignored. */
 } adpsgd_config;
 
 /* Schedules (Algorithm 1: kind 0; Algorithm 2: kind 1; kind 2: a piecewise-constant period,

@@ -125,6 +125,73 @@ __global__ void __launch_bounds__(kThreads, (NMAX >= 16 ? 1 : 2)) sync_step_kern
 
 using SyncStepKernel = void (*)(const SyncStepParams);
 
+// 9..16 replicas with Philox noise: the replicas in two halves of up to 8.  For each half the
+// thread loads x and v into registers, draws the half's normals in a rolled loop into its
+// shared-memory slots, applies the update, writes v and puts the new x into the same slots.
+// The averaging then takes the n new values of the group from shared memory.  Registers hold
+// one half at a time, so 4 blocks of 128 threads (16 warps) fit per SM where the 16-replica
+// register form fits 8 warps.  Same operations and order as sync_step_kernel.
+constexpr int kHalvesThreads = 128;
+constexpr int kHalf = 8;
+
+template <bool LOSS>
+__global__ void __launch_bounds__(kHalvesThreads, 4) sync_step_halves_kernel(const SyncStepParams p)
+{
+    // thread t, replica i: slots[t][i]; the pad row keeps the 16-byte accesses of 8 neighbouring
+    // threads on distinct banks
+    __shared__ float4 slots[kHalvesThreads][2 * kHalf + 1];
+    const AvgParams& a = p.avg;
+    const float nf = (float)a.n;
+    const bool wd = p.wd != 0.0f;
+    const int t = threadIdx.x;
+    double accD = 0.0, accL = 0.0;
+    bool redo = false;
+    const int64_t stride = (int64_t)gridDim.x * kHalvesThreads;
+    for (int64_t q = (int64_t)blockIdx.x * kHalvesThreads + t; q < a.Q; q += stride) {
+        const float4 hv = __ldg(reinterpret_cast<const float4*>(a.h) + q);
+        const float4 cv = __ldg(reinterpret_cast<const float4*>(a.c) + q);
+#pragma unroll 1
+        for (int r0 = 0; r0 < a.n; r0 += kHalf) {
+            float4 xv[kHalf], vv[kHalf];
+#pragma unroll
+            for (int u = 0; u < kHalf; ++u)
+                if (r0 + u < a.n) {
+                    const int64_t row = (int64_t)(r0 + u) * a.P;
+                    xv[u] = reinterpret_cast<const float4*>(a.x + row)[q];
+                    vv[u] = reinterpret_cast<const float4*>(p.v + row)[q];
+                }
+#pragma unroll 1
+            for (int i = r0; i < a.n && i < r0 + kHalf; ++i)
+                slots[t][i] = normals4(p.keys, (uint32_t)q + p.q0, (uint32_t)i, p.k, 0u);
+#pragma unroll
+            for (int u = 0; u < kHalf; ++u)
+                if (r0 + u < a.n) {
+                    const float4 z = slots[t][r0 + u];
+                    if (wd) {
+                        sgd_update<true>(xv[u].x, vv[u].x, hv.x, cv.x, z.x, p.gamma, p.mu, p.wd, p.sigma);
+                        sgd_update<true>(xv[u].y, vv[u].y, hv.y, cv.y, z.y, p.gamma, p.mu, p.wd, p.sigma);
+                        sgd_update<true>(xv[u].z, vv[u].z, hv.z, cv.z, z.z, p.gamma, p.mu, p.wd, p.sigma);
+                        sgd_update<true>(xv[u].w, vv[u].w, hv.w, cv.w, z.w, p.gamma, p.mu, p.wd, p.sigma);
+                    } else {
+                        sgd_update<false>(xv[u].x, vv[u].x, hv.x, cv.x, z.x, p.gamma, p.mu, p.wd, p.sigma);
+                        sgd_update<false>(xv[u].y, vv[u].y, hv.y, cv.y, z.y, p.gamma, p.mu, p.wd, p.sigma);
+                        sgd_update<false>(xv[u].z, vv[u].z, hv.z, cv.z, z.z, p.gamma, p.mu, p.wd, p.sigma);
+                        sgd_update<false>(xv[u].w, vv[u].w, hv.w, cv.w, z.w, p.gamma, p.mu, p.wd, p.sigma);
+                    }
+                    reinterpret_cast<float4*>(p.v + (int64_t)(r0 + u) * a.P)[q] = vv[u];
+                    slots[t][r0 + u] = xv[u];
+                }
+        }
+        redo |= !finish_group<2 * kHalf, true, LOSS, true, true>(a, q, slots[t], nf, accD, accL);
+    }
+    if (redo)
+        for (int64_t q = (int64_t)blockIdx.x * kHalvesThreads + t; q < a.Q; q += stride)
+            redo_group<true, LOSS, true>(a, q, nf, accD, accL);
+    finish_sums_n<LOSS, kHalvesThreads>(a, accD, accL);
+}
+
+bool use_halves(int32_t n, bool bf16) { return !bf16 && n > kHalf && n <= 2 * kHalf; }
+
 template <int NMAX>
 SyncStepKernel pick_nmax(bool bf16, bool loss)
 {
@@ -132,9 +199,11 @@ SyncStepKernel pick_nmax(bool bf16, bool loss)
     return loss ? sync_step_kernel<NMAX, false, true> : sync_step_kernel<NMAX, false, false>;
 }
 
-// 9..16 replicas: the bf16 noise tensor only (sync_step_supported).
+// 9..16 replicas: the two-halves form with Philox noise, the 16-replica register form with the
+// bf16 noise tensor.
 SyncStepKernel pick(int32_t n, bool bf16, bool loss)
 {
+    if (use_halves(n, bf16)) return loss ? sync_step_halves_kernel<true> : sync_step_halves_kernel<false>;
     if (n <= 2) return pick_nmax<2>(bf16, loss);
     if (n <= 4) return pick_nmax<4>(bf16, loss);
     if (n <= 8) return pick_nmax<8>(bf16, loss);
@@ -143,29 +212,28 @@ SyncStepKernel pick(int32_t n, bool bf16, bool loss)
 
 }  // namespace
 
-// Used where it measured faster than the two kernels it replaces: up to 8 replicas, and up to 16
-// with the pre-materialised bf16 noise.  With Philox noise and 9..16 replicas the 16-replica form
-// (one block of 256 per SM, 234 registers, the generator loop included) measured 0.54-0.62 of
-// the copy peak at n = 9 and 12 against 0.56-0.64 for the two kernels from P = 2^22 to 2^26, and
-// 0.61-0.66 against 0.60-0.63 at n = 16.
+// Every shape it takes measured faster than the two kernels it replaces.  With Philox noise and
+// 9..16 replicas the two-halves form measured 0.69-0.76 of the copy peak at n = 9, 0.77-0.83 at
+// n = 12 and 0.83-0.89 at n = 16 (P = 2^22 to 2^26), against 0.56-0.64 for the two kernels; the
+// 16-replica register form (one block of 256 per SM, 234 registers) had measured 0.54-0.66 there.
 bool sync_step_supported(int32_t n, int64_t P, const void* x, const void* v, const void* h, const void* c,
                          const void* noise_bf16)
 {
     auto al = [](const void* ptr, unsigned mask) { return (reinterpret_cast<uintptr_t>(ptr) & mask) == 0; };
-    const int max_n = noise_bf16 != nullptr ? kSyncStepMaxReplicas : 8;
-    return n >= 1 && n <= max_n && P % 4 == 0 && al(x, 15) && al(v, 15) && al(h, 15) && al(c, 15) &&
+    return n >= 1 && n <= kSyncStepMaxReplicas && P % 4 == 0 && al(x, 15) && al(v, 15) && al(h, 15) && al(c, 15) &&
            (noise_bf16 == nullptr || al(noise_bf16, 7));
 }
 
 int sync_step_grid(int32_t n, int64_t P, bool bf16, bool loss, int sms)
 {
+    const int threads = use_halves(n, bf16) ? kHalvesThreads : kThreads;
     int per_sm = 0;
-    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, pick(n, bf16, loss), kThreads, 0) != cudaSuccess ||
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, pick(n, bf16, loss), threads, 0) != cudaSuccess ||
         per_sm < 1) {
         cudaGetLastError();
         per_sm = 1;
     }
-    const int64_t work = (P / 4 + kThreads - 1) / kThreads;
+    const int64_t work = (P / 4 + threads - 1) / threads;
     int64_t grid = (int64_t)per_sm * sms;
     if (grid > work) grid = work;
     if (grid < 1) grid = 1;
@@ -195,7 +263,7 @@ cudaError_t launch_sync_step(const SyncStepArgs& s, cudaStream_t stream)
     p.sigma = s.sigma;
     p.keys = *s.keys;
     const SyncStepKernel kernel = pick(s.n, s.noise_bf16 != nullptr, s.loss);
-    kernel<<<(unsigned)s.grid, kThreads, 0, stream>>>(p);
+    kernel<<<(unsigned)s.grid, use_halves(s.n, s.noise_bf16 != nullptr) ? kHalvesThreads : kThreads, 0, stream>>>(p);
     return cudaGetLastError();
 }
 

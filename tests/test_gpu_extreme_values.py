@@ -122,13 +122,14 @@ def test_identical_replicas_give_exact_zero():
     assert _same_bits(_host(xd), x)
 
 
-@pytest.mark.parametrize("n", [4, 6])
+@pytest.mark.parametrize("n", [4, 6, 12])
 @pytest.mark.parametrize("kind", ["tiny", "huge"])
 @pytest.mark.parametrize("mode", ["unfused", "intervals", "sync_step"])
 def test_run_at_extreme_scales(kind, mode, n):
     # A short CPSGD run whose steps and syncs stay at the scale of the data: tiny values with tiny
     # noise (every sum subnormal), or huge values whose squares leave fp32.  Six replicas run the
-    # kernels built for up to 8 with two slots unused, four those built for exactly 4.
+    # kernels built for up to 8 with two slots unused, four those built for exactly 4, and twelve
+    # the fused step's two-halves form, whose averaging reads the new x from shared memory.
     K, p = 6, 2
     P = 1032 if mode == "sync_step" else 1031  # the fused sync step takes P % 4 == 0 only
     x, h, c = _problem(n, P, kind, seed=5)
