@@ -389,8 +389,10 @@ int adpsgd_noise_fill_bf16(uint64_t seed, int32_t n, int64_t P, uint16_t* out, v
  * managed memory, another device's memory, and host memory that is not page-locked go through
  * cudaMemcpyAsync.  The device side must be device (or managed) memory.  Both pointers 16-byte
  * aligned; bytes need not be a multiple of 16.
- * bytes == 0 does nothing.  The caller keeps both buffers alive until the stream has passed
- * the copy.
+ * bytes == 0 does nothing.  Both buffers must hold `bytes` bytes from the given addresses: the
+ * library cannot check a buffer's length, and a page-locked host buffer shorter than `bytes`
+ * makes the copy kernel read or write past its mapping (a device fault).  The caller keeps both
+ * buffers alive until the stream has passed the copy.
  * Errors: E_INVAL (NULL pointer with bytes > 0, bytes < 0, the device side not device memory,
  * the host side device memory), E_ALIGN, E_CUDA. */
 int adpsgd_copy_h2d(void* dst, const void* src, int64_t bytes, void* stream);
