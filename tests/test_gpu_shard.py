@@ -104,6 +104,7 @@ def _rel(a, b):
     (8, 1 << 18, 2, False, "sync_step", False),         # the bench's launch form
     (4, 4 * 777, 4, False, "intervals", False),
     (16, 4 * 2049, 2, True, "sync_step", False),        # bf16 noise tensor filled per shard
+    (12, 4 * 3001, 3, False, "sync_step", False),       # the two-halves form of the fused step
 ])
 def test_sharded_run_equals_unsharded_run(n, P, g, bf16, mode, track):
     K = 48
