@@ -38,7 +38,9 @@ struct SyncStepParams {
 // at n = 8, P = 2^26, 0.90 against 0.81 at 2^24 and 0.93 against 0.87 at n = 4, P = 2^26.  The
 // two-halves form below, with halves of 4 at 5 or 6 blocks of 128 per SM (92 or 80 registers),
 // measured 0.85-0.86 at n = 8, P = 2^26 and 0.80 at n = 6, against 0.93 and 0.88 here; the
-// generator loop unrolled by two (two replicas' chains interleaved) measured 0.5-1.5 % slower.
+// generator loop unrolled by two (two replicas' chains interleaved) measured 0.5-1.5 % slower,
+// and v staged in shared memory by per-thread cp.async copies while the generator runs (79-96
+// registers: 2 or 3 blocks of 256, or 5 or 6 of 128 per SM) 0.80-0.90 against 0.92 at n = 8.
 // Other forms measured slower on resnet18-n8 than the unrolled form did at the time (0.314 ms,
 // one launch under ncu, 225 M warp-instructions at 60 % issue; 0.294 ms and 213 M since the
 // generator's fma division and square root):
