@@ -108,6 +108,34 @@ def test_several_groups_per_thread(n):
     assert np.array_equal(host(vd).view(np.uint32), v.view(np.uint32))
 
 
+def test_two_halves_form_at_2_24_columns():
+    # 16 replicas with Philox noise take the two-halves form; at 2^24 columns every thread of its
+    # persistent grid takes dozens of column groups.  Every sync against the all-core oracle, and
+    # x, v bit-exact at the end.
+    n, P, K = 16, 1 << 24, 24
+    w = inputs.WORKLOADS["resnet18-n8"]
+    h, c = inputs.draw_h(P, w.h_dist, 11), inputs.draw_c(P, 1.0, 11)
+    x, v = inputs.random_state(n, P, 11)
+    xd, vd = dev(x), dev(v)
+    cfg = abi.make_config(n, P, momentum=0.9, weight_decay=5e-4, noise_sigma=0.8, seed=w.seed, fuse_sync_step=True)
+    sched = abi.make_schedule(abi.ADPSGD, K, 2, K_s=6, lr0=0.1)
+    tr = abi.TraceBuffers(K + 1)
+    with abi.adpsgd_init(cfg, xd, vd, dev(h), dev(c)) as ctx:
+        st = abi.adpsgd_run(ctx, sched, abi.adpsgd_state_init(sched), trace=tr)
+    # syncs one iteration apart (p = 1) keep the two kernels for the step enqueued ahead of a wait
+    assert st.sync_step_launches > 0 and st.sync_step_launches + st.average_launches == st.rounds
+    spec = O.ScheduleSpec(kind=abi.ADPSGD, K=K, p_init=2, K_s=6, lr0=0.1)
+    otr = O.run(x, v, h, c, spec=spec, seed=w.seed, mu=0.9, wd=5e-4, sigma=0.8, threads=O.host_threads())
+    g = tr.arrays()
+    assert np.array_equal(g["k"], otr.k) and np.array_equal(g["p"], otr.p) and np.array_equal(g["phase"], otr.phase)
+    for a, b in zip(g["S"], otr.S):
+        assert rel(a, b) < REL
+    for a, b in zip(g["loss"], otr.loss):
+        assert rel(a, b) < REL
+    assert np.array_equal(host(xd).view(np.uint32), x.view(np.uint32))
+    assert np.array_equal(host(vd).view(np.uint32), v.view(np.uint32))
+
+
 def test_fused_equals_unfused_at_a_larger_size():
     args = dict(n=8, P=(1 << 20) + 4 * 11, K=120, kind=abi.ADPSGD, p=4, K_s=30, milestones=(60, 90))
     a = _run(fused=False, **args)
