@@ -29,7 +29,9 @@ struct SyncStepParams {
     PhiloxKeys keys;
 };
 
-// Register cap: 128 per thread (2 blocks of 256 per SM) up to 8 replicas, 255 for 16.  One
+// Register cap: 128 per thread (2 blocks of 256 per SM) up to 8 replicas, 255 for 16, and 85 (3
+// blocks) for 3-4 replicas with Philox noise, which measured 0.90 against 0.87 of the copy peak at
+// n = 3, P = 2^26 (0.94 against 0.93 at n = 4); 2 replicas fit 3 blocks at the 128 cap.  One
 // thread per column group.  With Philox noise the n normals4 calls run first, in a loop that is
 // not unrolled, into per-thread shared-memory slots (NMAX x 256 float4 per block): the
 // generator's code is there once instead of n times, and its arithmetic runs while the loads of
@@ -72,7 +74,8 @@ struct SyncStepParams {
 //   under ncu, 306 M instructions (per-lane statistics, shuffles and h, c loads), 0.56 of the copy
 //   peak at n = 8, P = 2^26, and 0.45 with bf16 noise; 4 blocks per SM (64 registers) was slower.
 template <int NMAX, bool BF16, bool LOSS>
-__global__ void __launch_bounds__(kThreads, (NMAX >= 16 ? 1 : 2)) sync_step_kernel(const SyncStepParams p)
+__global__ void __launch_bounds__(kThreads, (NMAX >= 16 ? 1 : ((NMAX == 4 && !BF16) ? 3 : 2)))
+    sync_step_kernel(const SyncStepParams p)
 {
     __shared__ float4 zs[BF16 ? 1 : NMAX][BF16 ? 1 : kThreads];  // thread t's normals of replica i: zs[i][t]
     const AvgParams& a = p.avg;
