@@ -414,29 +414,33 @@ def run_gpu(args, w):
     k2_ms = kt2["average_ms"] / max(1, kt2["average_launches"])
     k2_gbs = k2_bytes / (k2_ms / 1000.0) / 1e9
 
-    # end to end through the C ABI from pinned host buffers (copies, run and read-back)
+    # End to end through the C ABI from pinned host buffers: the run's inputs as Algorithms 1 and
+    # 2 define them (one initial model w0 for every replica, momentum zero; h and c) in, the whole
+    # run, and its result out: the averaged model (one row) when the run ends with a sync, when
+    # every replica holds it, else every replica's row.
     e2e_value, h2d, d2h, e2e_phases = None, 0, 0, None
     if not args.no_e2e:
-        x0h = torch.zeros((n, P), dtype=torch.float32).pin_memory()
-        v0h = torch.zeros_like(x0h).pin_memory()
+        w0h = torch.zeros(P, dtype=torch.float32).pin_memory()  # x_0 = 0, this rank's columns
         hh = torch.from_numpy(h).pin_memory()
         ch = torch.from_numpy(c).pin_memory()
-        xout = torch.empty_like(x0h).pin_memory()
-        h2d = 4 * (2 * n * P_total + 2 * P_total)  # all ranks together
-        d2h = 4 * n * P_total
+        xout = torch.empty((n, P), dtype=torch.float32).pin_memory()
         ctx_e2e = context(fuse_sync_step=fuse_sync)  # set-up, outside the timed region
+        trace_e2e = abi.TraceBuffers(w.K + 1)
+        out_rows = [n]
 
         marks = [torch.cuda.Event(enable_timing=True) for _ in range(4)]
 
         def e2e_step():
-            # inputs in and the averaged parameters out through the library's transfer calls
             marks[0].record(stream)
-            for dst, src in ((xd, x0h), (vd, v0h), (hd, hh), (cd, ch)):
-                abi.adpsgd_copy_h2d(dst, src, stream=stream)
+            abi.adpsgd_init_replicas(ctx_e2e, w0h)
+            abi.adpsgd_copy_h2d(hd, hh, stream=stream)
+            abi.adpsgd_copy_h2d(cd, ch, stream=stream)
             marks[1].record(stream)
-            abi.adpsgd_run(ctx_e2e, sched, abi.adpsgd_state_init(sched))
+            abi.adpsgd_run(ctx_e2e, sched, abi.adpsgd_state_init(sched), trace=trace_e2e)
             marks[2].record(stream)
-            abi.adpsgd_copy_d2h(xout, xd, stream=stream)
+            ended_with_sync = trace_e2e.len > 0 and int(trace_e2e.k[trace_e2e.len - 1]) == w.K - 1
+            out_rows[0] = 1 if ended_with_sync else n
+            abi.adpsgd_copy_d2h(xout, xd, 4 * out_rows[0] * P, stream=stream)
             marks[3].record(stream)
 
         e2e_step()
@@ -451,6 +455,8 @@ def run_gpu(args, w):
             marks[0].elapsed_time(marks[1]), marks[1].elapsed_time(marks[2]), marks[2].elapsed_time(marks[3])))
         dt = max_over_ranks(pg, (time.perf_counter() - t0) / e2e_steps, device)
         e2e_value = rp_per_step / dt
+        h2d = 4 * 3 * P_total  # all ranks together: w0, h and c
+        d2h = 4 * out_rows[0] * P_total
         e2e_phases = {"h2d_ms": marks[0].elapsed_time(marks[1]), "run_ms": marks[1].elapsed_time(marks[2]),
                       "d2h_ms": marks[2].elapsed_time(marks[3]), "wall_ms": dt * 1000.0}
         ctx_e2e.close()
@@ -533,6 +539,9 @@ def run_gpu(args, w):
                        "l2": "inputs larger than L2 (x, v = %.0f MB per rank)" % (8 * n * P / 1e6),
                        "parallelism": parallelism},
             "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+                    "copies": "in: the initial model w0 [P] (adpsgd_init_replicas: every replica set to it on "
+                              "the device, momentum zeroed), h and c; out: the averaged model [P] when the run "
+                              "ends with a sync, else every replica's row",
                     "last_step": e2e_phases},
             "gpu_launches": launches,
             "roofline": {"kernel": "local_step_kernel", "bound": "hbm", "achieved": k1_gbs, "peak": peak,

@@ -396,6 +396,16 @@ int adpsgd_noise_fill_bf16(uint64_t seed, int32_t n, int64_t P, uint16_t* out, v
  * Errors: E_INVAL (NULL pointer with bytes > 0, bytes < 0, the device side not device memory,
  * the host side device memory), E_ALIGN, E_CUDA. */
 int adpsgd_copy_h2d(void* dst, const void* src, int64_t bytes, void* stream);
+
+/* The initialisation of Algorithms 1 and 2: every replica starts from the same model,
+ * w_{0,i} = w_0, with zero momentum.  Sets each of the context's n rows of x to the P floats at
+ * w0 and v to zero, enqueued on the context's stream (a column shard passes its own P columns of
+ * w_0).  w0: fp32 [P], host or device memory, kept alive by the caller until the stream has
+ * passed the call; it may be a row of x.  Device memory of the current device and page-locked
+ * host memory are read once by a broadcast kernel (host memory through its mapped address, so a
+ * run's initial model crosses the host link once, not n times); other memory is first copied
+ * into row 0 of x by cudaMemcpyAsync.  Errors: E_INVAL (NULL), E_CUDA. */
+int adpsgd_init_replicas(adpsgd_ctx* ctx, const float* w0);
 int adpsgd_copy_d2h(void* dst, const void* src, int64_t bytes, void* stream);
 
 /* Device time of the kernels launched through ctx while cfg.time_kernels was set, summed from

@@ -116,6 +116,7 @@ _SIGS = {
     "adpsgd_shard_combine": (C.c_int, [C.POINTER(Shard), C.POINTER(C.c_double), C.c_int64, C.POINTER(C.c_double)]),
     "adpsgd_noise_fill_bf16_part": (C.c_int, [C.c_uint64, C.c_int32, C.c_int64, C.c_int32, C.c_int64, _P, _P]),
     "adpsgd_copy_h2d": (C.c_int, [_P, _P, C.c_int64, _P]),
+    "adpsgd_init_replicas": (C.c_int, [_P, _P]),
     "adpsgd_copy_d2h": (C.c_int, [_P, _P, C.c_int64, _P]),
     "adpsgd_kernel_times": (C.c_int, [_P, C.POINTER(KernelTiming)]),
     "adpsgd_reset_kernel_times": (C.c_int, [_P]),
@@ -403,6 +404,12 @@ def _nbytes(t, nbytes):
 def adpsgd_copy_h2d(dst, src, nbytes: int | None = None, stream=None) -> None:
     """Host tensor src -> device tensor dst (nbytes: all of src by default), enqueued on stream."""
     _check(load().adpsgd_copy_h2d(_ptr(dst), _ptr(src), _nbytes(src, nbytes), _stream(stream)), "adpsgd_copy_h2d")
+
+
+def adpsgd_init_replicas(ctx: Context, w0) -> None:
+    """Every replica row of x set to w0 (fp32 [P], host or device tensor) and v to zero, on the
+    context's stream."""
+    _check(load().adpsgd_init_replicas(ctx.handle, _ptr(w0)), "adpsgd_init_replicas")
 
 
 def adpsgd_copy_d2h(dst, src, nbytes: int | None = None, stream=None) -> None:

@@ -84,6 +84,9 @@ cudaError_t launch_sync_step(const SyncStepArgs& a, cudaStream_t stream);
 // bytes from src to dst by a copy kernel on `stream`.  Both are device addresses (for host
 // memory: the mapped device address of a page-locked buffer), 16-byte aligned.
 cudaError_t launch_copy(void* dst, const void* src, int64_t bytes, int sms, cudaStream_t stream);
+// dst rows [0, rows) of P floats each (row stride P) = the P floats at src, a device address (for
+// host memory: the mapped device address of a page-locked buffer); src may be one of dst's rows.
+cudaError_t launch_broadcast_rows(float* dst, const float* src, int32_t rows, int64_t P, int sms, cudaStream_t stream);
 
 // Fixed device scratch (no allocation): partial sums for up to static_scratch_max_blocks()
 // blocks, the two finished sums and the completion counter.  The first call on a device looks the address up.

@@ -1055,6 +1055,41 @@ int transfer(void* dst, const void* src, int64_t bytes, void* stream, bool to_de
 
 }  // namespace
 
+int adpsgd_init_replicas(adpsgd_ctx* ctx, const float* w0)
+{
+    if (ctx == nullptr || w0 == nullptr) return ADPSGD_E_INVAL;
+    NvtxRange range("adpsgd_init_replicas");
+    const int32_t n = ctx->cfg.n;
+    const int64_t P = ctx->cfg.P;
+    const size_t row_bytes = (size_t)P * sizeof(float);
+    cudaMemoryType type;
+    int dev = -1;
+    cudaError_t e = memory_type(w0, &type, &dev);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaPointerGetAttributes");
+    // The kernel reads w0 where it is device memory of this device or page-locked host memory
+    // (through its mapped address); anything else is first copied into row 0 of x.
+    const float* src = nullptr;
+    int32_t first = 0;
+    void* mapped = nullptr;
+    if (type == cudaMemoryTypeDevice && dev == ctx->device) {
+        src = w0;
+    } else if (type == cudaMemoryTypeHost &&
+               cudaHostGetDevicePointer(&mapped, const_cast<float*>(w0), 0) == cudaSuccess) {
+        src = static_cast<const float*>(mapped);
+    } else {
+        cudaGetLastError();  // a failed cudaHostGetDevicePointer leaves no sticky error
+        e = cudaMemcpyAsync(ctx->x, w0, row_bytes, cudaMemcpyDefault, ctx->stream);
+        if (e != cudaSuccess) return cuda_fail(e, "cudaMemcpyAsync");
+        src = ctx->x;
+        first = 1;
+    }
+    e = adpsgd::launch_broadcast_rows(ctx->x + (int64_t)first * P, src, n - first, P, ctx->sms, ctx->stream);
+    if (e != cudaSuccess) return cuda_fail(e, "broadcast kernel");
+    e = cudaMemsetAsync(ctx->v, 0, (size_t)n * row_bytes, ctx->stream);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaMemsetAsync");
+    return ADPSGD_OK;
+}
+
 int adpsgd_copy_h2d(void* dst, const void* src, int64_t bytes, void* stream)
 {
     return transfer(dst, src, bytes, stream, true);

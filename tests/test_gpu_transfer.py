@@ -151,3 +151,84 @@ def test_run_fed_and_read_back_through_the_transfer_calls():
     g = tr.arrays()
     assert np.array_equal(g["k"], otr.k) and np.array_equal(g["p"], otr.p)
     assert np.array_equal(xo.numpy().view(np.uint32), x.view(np.uint32))
+
+
+def _w0(P, seed):
+    g = torch.Generator().manual_seed(seed)
+    return torch.randn(P, generator=g, dtype=torch.float32)
+
+
+@pytest.mark.parametrize("where", ["pinned", "pageable", "device", "row_of_x", "inner_row_of_x"])
+@pytest.mark.parametrize("n,P", [(1, 8), (3, 4099), (8, 1 << 20), (5, (1 << 18) + 4)])
+def test_init_replicas(where, n, P):
+    # Algorithms 1 and 2 start every replica from the same model with zero momentum: every row of
+    # x equals w0 bit for bit, v is zero, and nothing outside x and v is written.
+    w0 = _w0(P, n * 7 + P)
+    xbuf = torch.full((n * P + 64,), 3.5, dtype=torch.float32, device=DEV)
+    vbuf = torch.full((n * P + 64,), -1.25, dtype=torch.float32, device=DEV)
+    xd, vd = xbuf[:n * P].view(n, P), vbuf[:n * P].view(n, P)
+    z = torch.zeros(P, device=DEV)
+    if where == "pinned":
+        src = w0.pin_memory()
+    elif where == "pageable":
+        src = w0
+    elif where == "device":
+        src = w0.to(DEV)
+    else:
+        r = 0 if where == "row_of_x" else n - 1
+        xd[r].copy_(w0.to(DEV))
+        src = xd[r]
+    with abi.adpsgd_init(abi.make_config(n, P), xd, vd, z, z) as ctx:
+        abi.adpsgd_init_replicas(ctx, src)
+        torch.cuda.synchronize()
+    want = w0.numpy().view(np.uint32)
+    got = xd.cpu().numpy().view(np.uint32)
+    assert all(np.array_equal(got[i], want) for i in range(n))
+    assert bool((vd == 0).all()) and not bool(torch.signbit(vd).any())
+    assert bool((xbuf[n * P:] == 3.5).all()) and bool((vbuf[n * P:] == -1.25).all()), "wrote past x or v"
+
+
+def test_init_replicas_refuses_null():
+    n, P = 2, 64
+    xd, vd, z = torch.zeros((n, P), device=DEV), torch.zeros((n, P), device=DEV), torch.zeros(P, device=DEV)
+    with abi.adpsgd_init(abi.make_config(n, P), xd, vd, z, z) as ctx:
+        with pytest.raises(abi.AdpsgdError) as e:
+            abi.adpsgd_init_replicas(ctx, None)
+        assert e.value.status == abi.E_INVAL
+
+
+@pytest.mark.parametrize("kind", [abi.ADPSGD, abi.CPSGD])
+def test_run_from_one_initial_model_against_the_oracle(kind):
+    # The end-to-end form: one host row w0 broadcast to every replica (zero momentum), h and c
+    # copied in, a whole run, and the result read back: one row when the run ends with a sync
+    # (CPSGD p = 4 over 40 iterations does), every row otherwise.
+    w = inputs.WORKLOADS["quadratic-n4-P1M"]
+    n, P, K = w.n, (1 << 16) + 12, 40
+    h, c = inputs.problem(w, P)
+    w0 = _w0(P, 5)
+    hh, ch = torch.from_numpy(h).pin_memory(), torch.from_numpy(c).pin_memory()
+    xd, vd = torch.full((n, P), 7.0, device=DEV), torch.full((n, P), 7.0, device=DEV)
+    hd, cd = torch.empty(P, device=DEV), torch.empty(P, device=DEV)
+    abi.adpsgd_copy_h2d(hd, hh)
+    abi.adpsgd_copy_h2d(cd, ch)
+    cfg = abi.make_config(n, P, momentum=w.mu, weight_decay=w.wd, noise_sigma=w.sigma, seed=w.seed)
+    K_s = 10 if kind == abi.ADPSGD else 0
+    sched = abi.make_schedule(kind, K, 4, K_s=K_s, lr0=w.lr0)
+    tr = abi.TraceBuffers(K + 1)
+    with abi.adpsgd_init(cfg, xd, vd, hd, cd) as ctx:
+        abi.adpsgd_init_replicas(ctx, w0.pin_memory())
+        abi.adpsgd_run(ctx, sched, abi.adpsgd_state_init(sched), trace=tr)
+    g = tr.arrays()
+    one_row = g["k"][-1] == K - 1
+    assert one_row or kind == abi.ADPSGD
+    xo = torch.empty((1 if one_row else n, P), dtype=torch.float32).pin_memory()
+    abi.adpsgd_copy_d2h(xo, xd, xo.numel() * 4)
+    torch.cuda.synchronize()
+    x = np.repeat(w0.numpy()[None, :], n, axis=0)
+    v = np.zeros((n, P), np.float32)
+    spec = O.ScheduleSpec(kind=kind, K=K, p_init=4, K_s=K_s, lr0=w.lr0)
+    otr = O.run(x, v, h, c, spec=spec, seed=w.seed, mu=w.mu, wd=w.wd, sigma=w.sigma)
+    assert np.array_equal(g["k"], otr.k) and np.array_equal(g["p"], otr.p)
+    assert np.array_equal(xo.numpy().view(np.uint32), x[:xo.shape[0]].view(np.uint32))
+    assert np.array_equal(xd.cpu().numpy().view(np.uint32), x.view(np.uint32))
+    assert np.array_equal(vd.cpu().numpy().view(np.uint32), v.view(np.uint32))
