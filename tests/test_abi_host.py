@@ -106,6 +106,7 @@ def test_init_argument_checks_before_any_cuda_call():
     bf = abi.make_config(4, 1024, noise_mode=abi.NOISE_BF16)
     assert lib.adpsgd_init(C.byref(bf), 16, 32, 48, 64, None, None, C.byref(out)) == abi.E_INVAL
     assert lib.adpsgd_local_steps(None, 0, 1, None) == abi.E_INVAL
+    assert lib.adpsgd_init_replicas(None, 16) == abi.E_INVAL
     assert lib.adpsgd_philox_fill(0, 0, 1, 4, 0, None, None) == abi.E_INVAL
     assert lib.adpsgd_philox_fill(0, 0, 1, 4, 0, 8, None) == abi.E_ALIGN
     assert lib.adpsgd_philox_fill(0, 0, 1, 4, 1 << 32, 16, None) == abi.E_INVAL
