@@ -349,10 +349,12 @@ def run_gpu(args, w):
 
     sched = schedule_for(abi, w)
     ctx = context(time_kernels=TIMING_PERIOD, fuse_sync_step=fuse_sync)
+    w0d = torch.zeros(P, dtype=torch.float32, device=device)  # x_0 = 0, the initial model on the device
 
     def one_run():
-        xd.zero_()
-        vd.zero_()
+        # Algorithm 2 from the start: every replica set to w0 and the momentum zeroed by the
+        # library (one broadcast kernel and a memset), then the whole run.
+        abi.adpsgd_init_replicas(ctx, w0d)
         st = abi.adpsgd_state_init(sched)
         return abi.adpsgd_run(ctx, sched, st)
 
@@ -378,7 +380,8 @@ def run_gpu(args, w):
         for _ in range(args.steps):
             stats = one_run()
             rounds.append(stats.rounds)
-            launches += stats.local_step_launches + stats.average_launches + stats.sync_step_launches
+            # the broadcast kernel of the initialisation, then the run's kernels
+            launches += 1 + stats.local_step_launches + stats.average_launches + stats.sync_step_launches
         ev1.record(stream)
         torch.cuda.synchronize(device)
         barrier(pg, device)
@@ -466,8 +469,7 @@ def run_gpu(args, w):
     if not args.no_fused and n <= 32:
         with context(time_kernels=TIMING_PERIOD, fuse_intervals=True) as ctx_f:
             def fused_run():
-                xd.zero_()
-                vd.zero_()
+                abi.adpsgd_init_replicas(ctx_f, w0d)
                 return abi.adpsgd_run(ctx_f, sched, abi.adpsgd_state_init(sched))
             fused_run()
             abi.adpsgd_reset_kernel_times(ctx_f)
@@ -492,8 +494,7 @@ def run_gpu(args, w):
     comparison = None
     if not args.no_compare:
         tr_a = abi.TraceBuffers(w.K + 1)
-        xd.zero_()
-        vd.zero_()
+        abi.adpsgd_init_replicas(ctx, w0d)
         sa = abi.adpsgd_run(ctx, sched, abi.adpsgd_state_init(sched), trace=tr_a)
         ta = tr_a.arrays()
         p_eq = max(1, round(w.K / max(1, sa.rounds)))
@@ -503,8 +504,7 @@ def run_gpu(args, w):
                 continue
             sc = abi.make_schedule(abi.CPSGD, w.K, p_c, lr0=w.lr0, lr_factor=w.lr_factor, milestones=w.milestones)
             tr_c = abi.TraceBuffers(w.K + 1)
-            xd.zero_()
-            vd.zero_()
+            abi.adpsgd_init_replicas(ctx, w0d)
             st_c = abi.adpsgd_run(ctx, sc, abi.adpsgd_state_init(sc), trace=tr_c)
             rows[label] = (sc, st_c, tr_c.arrays())
         comparison = {}
