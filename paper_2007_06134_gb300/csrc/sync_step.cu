@@ -139,7 +139,9 @@ using SyncStepKernel = void (*)(const SyncStepParams);
 // The averaging then takes the n new values of the group from shared memory.  Registers hold
 // one half at a time, so 4 blocks of 128 threads (16 warps) fit per SM where the 16-replica
 // register form fits 8 warps.  Same operations and order as sync_step_kernel.  Balanced halves
-// (n = 9 as 5 + 4, 12 as 6 + 6) measured 1-3 % slower than 8 first.
+// (n = 9 as 5 + 4, 12 as 6 + 6) measured 1-3 % slower than 8 first.  With the bf16 noise tensor
+// this form (spilling a few registers) measured 0.87-0.95 against 0.90-0.96 for the 16-replica
+// register form, which has no generator to hide.
 constexpr int kHalvesThreads = 128;
 constexpr int kHalf = 8;
 
